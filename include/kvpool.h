@@ -1,0 +1,243 @@
+/*
+ * kvpool.h -- C ABI of libkvpool: one block-paged bf16 KV pool in HBM shared
+ * by many sequences (and several model layouts), the per-step append of each
+ * sequence's new K/V row, and batched paged decode attention over the pool.
+ *
+ * What the paper fixes and what it leaves to us
+ * ---------------------------------------------
+ * The paper (Maestro, a workload-aware scheduler for multi-agent LLM serving)
+ * treats this path as the engine under its runtime:
+ *   - KV footprint grows linearly with prompt + output length (§II, "KV cache
+ *     memory pressure"); per stage the runtime reserves alpha(M) * (P + L^)
+ *     of it (Eq. 2).
+ *   - One GPU's KV lives in a single shared pool whose pages are handed out
+ *     on demand to the stages of co-located models; when physical memory runs
+ *     out the stage is rejected, not crashed (§III-C, "Spatial multiplexing
+ *     with virtual-memory KV cache"; explicit accounting M_kv + M_res <= M_total).
+ *   - The serving engine pages the cache into fixed-size blocks reached
+ *     through a per-sequence block table (PagedAttention, §II and §IV-A).
+ *   - Decode dominates latency for long outputs (§II, "LLM inference cost
+ *     model"): every step, every live sequence attends with one new query over
+ *     its whole cached context.
+ * The paper gives no API, no layout and no kernel; those are this library's.
+ *
+ * Conventions (all entry points)
+ * ------------------------------
+ *   - Every function returns an int: KV_OK (0) or a negative kv_status.
+ *   - The caller owns ALL device memory (pool, tables, lengths, q, out,
+ *     workspace, error word) and all streams; pointers are plain device
+ *     addresses and cudaStream_t handles passed as void*.  The library owns only
+ *     host-side metadata (free lists, refcounts).
+ *   - Launches are asynchronous on the given stream (NULL = legacy default
+ *     stream).  Argument errors are detected on the host before anything is
+ *     launched and leave every buffer untouched.
+ *   - bf16 tensors are IEEE bfloat16 bit patterns (uint16), row-major and
+ *     contiguous.  Outputs are rounded fp32 -> bf16 to nearest-even.
+ *   - Out-of-range indices found on the device (a table entry outside the
+ *     pool, a context length beyond the table) never fault: the access is
+ *     skipped, the error word is set to KV_ERR_DEVICE_BOUNDS, and the results
+ *     of the affected sequence are unspecified.  Read it with
+ *     kv_pool_get_error().
+ *
+ * Pool layout
+ * -----------
+ * The pool is cut into pages of page_bytes.  A block of layout L (Hkv KV
+ * heads, head dim d, block size bs tokens) occupies block_bytes(L) =
+ * 2 * Hkv * bs * d * 2 bytes = k_L consecutive pages, and is named by the id
+ * of its first page.  Block id b starts at byte b * page_bytes and holds
+ *     [K|V][Hkv][bs][d]  (bf16),
+ * so the K (or V) tile of one KV head is one contiguous bs*d*2-byte run.
+ * Token j of a sequence lives in block table[s][j / bs] at offset j % bs.
+ */
+#ifndef KVPOOL_H
+#define KVPOOL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum kv_status {
+    KV_OK = 0,
+    KV_ERR_INVALID_ARG = -1,   /* bad pointer, size, id or layout; nothing launched */
+    KV_ERR_OUT_OF_BLOCKS = -2, /* allocation cannot be met; nothing allocated */
+    KV_ERR_CUDA = -3,          /* a CUDA runtime call failed */
+    KV_ERR_DEVICE_BOUNDS = -4, /* (error word) a device-side index check failed */
+    KV_ERR_UNSUPPORTED = -5,   /* shape not built into this library (d, G) */
+    KV_ERR_WORKSPACE = -6,     /* workspace missing or smaller than kv_workspace_bytes() */
+    KV_ERR_DEVICE_TIMEOUT = -7 /* (error word) a bounded device wait gave up */
+} kv_status;
+
+#define KV_MAX_LAYOUTS 4
+
+/* Geometry of one model's layer KV in the pool. */
+typedef struct kv_layout {
+    int32_t num_kv_heads; /* Hkv >= 1 */
+    int32_t head_dim;     /* d: 64 or 128 */
+} kv_layout;
+
+typedef struct kv_pool_desc {
+    void *device_base;     /* caller-owned device buffer, 256-byte aligned */
+    uint64_t pool_bytes;   /* its size; pages = pool_bytes / page_bytes */
+    int32_t block_size;    /* bs: tokens per block, 1..256, same for all layouts */
+    int32_t num_layouts;   /* 1..KV_MAX_LAYOUTS */
+    kv_layout layouts[KV_MAX_LAYOUTS];
+    uint64_t page_bytes;   /* 0 = smallest layout block; every layout's block
+                              bytes must be a multiple of it, and it a multiple of 256 */
+    int32_t *device_error; /* caller-owned device int32, zero-initialised */
+    uint64_t shuffle_seed; /* 0: free list hands out ascending ids; otherwise the
+                              initial free order is a seeded permutation
+                              (splitmix64 Fisher-Yates) to scatter placement */
+} kv_pool_desc;
+
+typedef struct kv_pool kv_pool;
+
+typedef struct kv_stats {
+    int64_t pages_total;
+    int64_t pages_unassigned;                /* whole free superpages */
+    int64_t blocks_used[KV_MAX_LAYOUTS];     /* blocks with refcount > 0 */
+    int64_t blocks_cached[KV_MAX_LAYOUTS];   /* free blocks held by the layout */
+    int64_t blocks_capacity[KV_MAX_LAYOUTS]; /* used + cached + unassigned/k */
+    uint64_t bytes_used;                     /* sum of used blocks' bytes */
+    uint64_t bytes_total;                    /* pages_total * page_bytes */
+} kv_stats;
+
+/* ---------------------------------------------------------------- pool --- */
+
+/*
+ * Create the host-side manager of a caller-owned device pool (§III-C: one
+ * shared KV pool per GPU, pages handed out per stage).  Allocation is a slab
+ * scheme: pages are grouped into superpages of K = max_L k_L pages; a layout
+ * takes a whole free superpage when its own free list is empty and cuts it
+ * into K / k_L blocks.  Freed blocks go back to their layout's LIFO free list.
+ * Also queries the current device (SM count) for launch sizing.
+ * Errors: KV_ERR_INVALID_ARG (null/misaligned pointers, bad geometry, pool
+ * smaller than one superpage), KV_ERR_CUDA.
+ */
+int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool);
+
+/* Release host metadata.  The device buffer is the caller's. */
+int kv_pool_destroy(kv_pool *pool);
+
+/*
+ * Reserve n blocks of layout `layout` (Eq. 2's per-stage reservation is n =
+ * ceil((P + L^) / bs) blocks; the caller decides n).  Writes n block ids
+ * (refcount 1) to the host array out_ids.  All-or-nothing: on
+ * KV_ERR_OUT_OF_BLOCKS nothing is allocated (§III-C: a stage whose memory
+ * cannot be mapped is rejected).
+ */
+int kv_alloc_blocks(kv_pool *pool, int layout, int n, int32_t *out_ids);
+
+/*
+ * Drop one reference to each of n blocks (host array).  A block whose count
+ * reaches zero returns to its layout's free list.  Validated before anything
+ * changes: every id must be a live block of `layout` holding at least as many
+ * references as it appears in ids, else KV_ERR_INVALID_ARG.
+ */
+int kv_free_blocks(kv_pool *pool, int layout, int n, const int32_t *ids);
+
+/*
+ * Add one reference to each of n live blocks of `layout` (a prefix shared by
+ * reference by several block tables).  Validated first; KV_ERR_INVALID_ARG.
+ */
+int kv_block_ref(kv_pool *pool, int layout, int n, const int32_t *ids);
+
+/* Refcount of a block id (0 = free), or KV_ERR_INVALID_ARG for a bad id. */
+int kv_block_refcount(const kv_pool *pool, int32_t id, int32_t *out_count);
+
+/* Counters of the pool (host only). */
+int kv_pool_stats(const kv_pool *pool, kv_stats *out);
+
+/*
+ * Asynchronously copy the device error word into *host_code (host memory; use
+ * pinned memory for true asynchrony) and reset it to zero, on `stream`.  The
+ * value is valid after the stream reaches this point (e.g. after
+ * cudaStreamSynchronize).  0 means no device-side error since the last call.
+ */
+int kv_pool_get_error(kv_pool *pool, void *stream, int32_t *host_code);
+
+/* ------------------------------------------------------- block tables --- */
+
+/*
+ * Copy a block table and context lengths from host to device on `stream`:
+ * host_table int32 [S][max_blocks] -> dev_table, host_ctx_lens int32 [S] ->
+ * dev_ctx_lens.  Lengths are post-append (they include the token appended this
+ * step).  Every entry a sequence can reach (the first ceil(len / bs) of its
+ * row) is checked on the host to be a whole block of `layout` inside the pool,
+ * and len <= max_blocks * bs; otherwise KV_ERR_INVALID_ARG and nothing is
+ * copied.  Entries past a sequence's last block are not read by any kernel.
+ * The copy is a cudaMemcpyAsync from the caller's host buffers: they must stay
+ * unchanged until the stream passes this point (pageable memory makes the call
+ * synchronous).
+ */
+int kv_block_table_upload(kv_pool *pool, int layout, const int32_t *host_table, int S,
+                          int max_blocks, const int32_t *host_ctx_lens, int32_t *dev_table,
+                          int32_t *dev_ctx_lens, void *stream);
+
+/* -------------------------------------------------------------- kernels --- */
+
+/*
+ * Append one token per sequence (the decode step writes the new token's K/V
+ * before attending, §II): for s < S with n = dev_ctx_lens[s] > 0 and every KV
+ * head g, copy k_new[s][g][:] and v_new[s][g][:] (bf16 [S][Hkv][d] device
+ * arrays) bit-exactly into slot (table[s][(n-1)/bs], (n-1) % bs).  Sequences
+ * with n <= 0 are skipped.  Device bounds failures skip the row and set the
+ * error word.
+ */
+int kv_append(kv_pool *pool, int layout, const uint16_t *k_new, const uint16_t *v_new,
+              const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks, int S,
+              void *stream);
+
+/*
+ * Bytes of device workspace paged_decode_attn needs for these sizes and this
+ * num_splits.  The workspace holds per-(sequence, KV head) arrival counters
+ * followed by fp32 split partials; its counter area must be zero before the
+ * first call that uses it (allocate it zero-filled, or call
+ * kv_workspace_clear once); every call that completes leaves it zero again.
+ */
+int kv_workspace_bytes(const kv_pool *pool, int layout, int S, int Hq, int max_blocks,
+                       int num_splits, size_t *out_bytes);
+
+/* Zero a workspace on `stream` (cudaMemsetAsync). */
+int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Batched paged decode attention.  For every sequence s < S (post-append
+ * length n = dev_ctx_lens[s]), every query head h < Hq and its KV head
+ * g = floor(h / G), G = Hq / Hkv (contiguous head groups):
+ *     out[s][h] = sum_{j<n} softmax_j(scale * q[s][h] . K_j) V_j
+ * with K_j, V_j the rows of head g at position j, found through dev_table.
+ * q, out: bf16 [S][Hq][d] device arrays.  A sequence with n == 0 gets zeros.
+ * Arithmetic: fp32 products and accumulation, online softmax in base 2,
+ * bf16 output rounded to nearest-even.
+ * Work split: the KV range of each sequence is cut into chunks of whole
+ * blocks; num_splits == 0 picks one chunk size for the batch from the SM
+ * count and the total length; num_splits > 0 cuts every sequence into at
+ * most num_splits equal block-aligned chunks.  Chunk partials (max, sum,
+ * unnormalised output) are combined in fixed chunk order, so results do not
+ * depend on where blocks sit in the pool.
+ * Errors: KV_ERR_INVALID_ARG, KV_ERR_UNSUPPORTED (d not 64/128, G not in
+ * {1,2,3,4,5,6,8}), KV_ERR_WORKSPACE.
+ */
+int paged_decode_attn(kv_pool *pool, int layout, const uint16_t *q, uint16_t *out,
+                      const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks,
+                      int S, int Hq, float scale, int num_splits, void *workspace,
+                      size_t ws_bytes, void *stream);
+
+/*
+ * Select the attention compute variant for later calls on this pool:
+ * 0 = automatic (the fastest measured for the shape), 1 = CUDA-core FMA,
+ * 2 = warp-level tensor-core MMA (mma.sync bf16, fp32 accumulate).
+ */
+int kv_set_attn_variant(kv_pool *pool, int variant);
+
+/* Library version string (static storage). */
+const char *kv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVPOOL_H */

@@ -1,0 +1,216 @@
+// kernels.cu -- KV append kernel and the launch wrappers of the C ABI
+// (kv_append, kv_workspace_bytes, paged_decode_attn).
+#include <cmath>
+#include <mutex>
+
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include "attn_launch.cuh"
+#include "pool_internal.h"
+
+namespace {
+
+// Append: the decode step writes the new token's K and V before attending
+// (§II).  One thread per 16-byte chunk of a (sequence, KV head, K|V) row; 16
+// consecutive threads write one 256-byte row (d = 128), so stores coalesce.
+__global__ void append_kernel(uint8_t *__restrict__ pool, const uint4 *__restrict__ k_new,
+                              const uint4 *__restrict__ v_new, const int32_t *__restrict__ table,
+                              const int32_t *__restrict__ ctx_lens, int32_t *err, int S, int Hkv, int D, int bs,
+                              int max_blocks, int64_t page_bytes, int64_t n_pages, int32_t pages_per_block)
+{
+    const int cpr = D / 8;  // 16-byte chunks per row
+    const int64_t total = (int64_t)S * Hkv * 2 * cpr;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(idx % cpr);
+        int64_t rest = idx / cpr;
+        const int kv = (int)(rest % 2);
+        rest /= 2;
+        const int g = (int)(rest % Hkv);
+        const int s = (int)(rest / Hkv);
+        const int32_t n = ctx_lens[s];
+        if (n <= 0) continue;
+        if (n > max_blocks * bs) {
+            atomicCAS(err, 0, KV_ERR_DEVICE_BOUNDS);
+            continue;
+        }
+        const int pos = n - 1;
+        const int32_t phys = table[(int64_t)s * max_blocks + pos / bs];
+        if (phys < 0 || (int64_t)phys + pages_per_block > n_pages) {
+            atomicCAS(err, 0, KV_ERR_DEVICE_BOUNDS);
+            continue;
+        }
+        const uint4 *src = (kv ? v_new : k_new) + ((int64_t)s * Hkv + g) * cpr + c;
+        uint8_t *dst = pool + (int64_t)phys * page_bytes +
+                       ((((int64_t)kv * Hkv + g) * bs + (pos % bs)) * D + (int64_t)c * 8) * 2;
+        *reinterpret_cast<uint4 *>(dst) = *src;
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// The pool seen as a 2-D bf16 tensor of rows of d elements; a box is 64
+// columns x 16 rows with the 128-byte swizzle, i.e. one half of a 16-token
+// K or V tile of one head.
+int ensure_tmap(kv_pool *p, int layout)
+{
+    std::lock_guard<std::mutex> g(p->mu);
+    if (p->tmap_ok[layout]) return KV_OK;
+    auto enc = encode_fn();
+    if (!enc) return KV_ERR_CUDA;
+    const int D = p->desc.layouts[layout].head_dim;
+    const uint64_t rows = (uint64_t)p->n_pages * p->page_bytes / ((uint64_t)D * 2);
+    cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)kvp::kTile};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&p->tmap[layout], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p->desc.device_base, dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return KV_ERR_CUDA;
+    p->tmap_ok[layout] = true;
+    return KV_OK;
+}
+
+bool aligned16(const void *ptr) { return ((uintptr_t)ptr & 15u) == 0; }
+
+int pick_variant(const kv_pool *p, int G)
+{
+    if (p->attn_variant) return p->attn_variant;
+    (void)G;
+    return 2;
+}
+
+// common argument checks of paged_decode_attn / kv_workspace_bytes
+int attn_shape(const kv_pool *p, int layout, int S, int Hq, int max_blocks, int *G_out)
+{
+    if (!p || layout < 0 || layout >= p->desc.num_layouts) return KV_ERR_INVALID_ARG;
+    if (S < 0 || max_blocks < 1 || Hq < 1) return KV_ERR_INVALID_ARG;
+    const kv_layout &L = p->desc.layouts[layout];
+    if (Hq % L.num_kv_heads) return KV_ERR_INVALID_ARG;
+    const int G = Hq / L.num_kv_heads;
+    if (L.head_dim != 64 && L.head_dim != 128) return KV_ERR_UNSUPPORTED;
+    if (p->desc.block_size % kvp::kTile) return KV_ERR_UNSUPPORTED;
+    if (!(G == 1 || G == 2 || G == 4 || G == 5 || G == 8)) return KV_ERR_UNSUPPORTED;
+    // unit ids and pool rows are 32-bit on the device
+    const int64_t tiles = ((int64_t)max_blocks * p->desc.block_size + kvp::kTile - 1) / kvp::kTile;
+    if ((int64_t)S * tiles * L.num_kv_heads >= INT32_MAX) return KV_ERR_INVALID_ARG;
+    if ((int64_t)p->n_pages * (int64_t)p->page_bytes / (2 * L.head_dim) >= INT32_MAX) return KV_ERR_INVALID_ARG;
+    if ((int64_t)max_blocks * p->desc.block_size >= INT32_MAX) return KV_ERR_INVALID_ARG;
+    *G_out = G;
+    return KV_OK;
+}
+
+int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sms,
+             cudaStream_t st, bool launch, int *P_out)
+{
+    if (D == 64) return kvp_attn_d64(variant, G, tmap, a, P_req, sms, st, launch, P_out);
+    return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, launch, P_out);
+}
+
+size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
+{
+    const size_t cnt = ((size_t)S * Hkv * 4 + 255) / 256 * 256;
+    *part_off = cnt;
+    return cnt + ((size_t)S * Hkv + (size_t)P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
+}
+
+}  // namespace
+
+extern "C" {
+
+int kv_append(kv_pool *p, int layout, const uint16_t *k_new, const uint16_t *v_new, const int32_t *dev_table,
+              const int32_t *dev_ctx_lens, int max_blocks, int S, void *stream)
+{
+    if (!p || layout < 0 || layout >= p->desc.num_layouts || S < 0 || max_blocks < 1) return KV_ERR_INVALID_ARG;
+    if (S == 0) return KV_OK;
+    if (!k_new || !v_new || !dev_table || !dev_ctx_lens) return KV_ERR_INVALID_ARG;
+    if (!aligned16(k_new) || !aligned16(v_new)) return KV_ERR_INVALID_ARG;
+    const kv_layout &L = p->desc.layouts[layout];
+    if (L.head_dim % 8) return KV_ERR_UNSUPPORTED;
+    const int64_t total = (int64_t)S * L.num_kv_heads * 2 * (L.head_dim / 8);
+    const int threads = 256;
+    const int64_t want = (total + threads - 1) / threads;
+    const int blocks = (int)std::min<int64_t>(want, (int64_t)std::max(1, p->sm_count) * 16);
+    append_kernel<<<blocks, threads, 0, (cudaStream_t)stream>>>(
+        (uint8_t *)p->desc.device_base, reinterpret_cast<const uint4 *>(k_new), reinterpret_cast<const uint4 *>(v_new),
+        dev_table, dev_ctx_lens, p->desc.device_error, S, L.num_kv_heads, L.head_dim, p->desc.block_size, max_blocks,
+        (int64_t)p->page_bytes, p->n_pages, p->pages_per_block[layout]);
+    return cudaGetLastError() == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+}
+
+int kv_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int max_blocks, int num_splits,
+                       size_t *out_bytes)
+{
+    int G = 0;
+    if (!out_bytes || num_splits < 0) return KV_ERR_INVALID_ARG;
+    int rc = attn_shape(p, layout, S, Hq, max_blocks, &G);
+    if (rc) return rc;
+    const kv_layout &L = p->desc.layouts[layout];
+    kvp::AttnArgs a{};
+    a.S = S;
+    a.Hkv = L.num_kv_heads;
+    int P = 0;
+    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, false, &P);
+    if (rc) return rc;
+    size_t off;
+    *out_bytes = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &off);
+    return KV_OK;
+}
+
+int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, const int32_t *dev_table,
+                      const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale, int num_splits,
+                      void *workspace, size_t ws_bytes, void *stream)
+{
+    int G = 0;
+    if (num_splits < 0 || !std::isfinite(scale)) return KV_ERR_INVALID_ARG;
+    int rc = attn_shape(p, layout, S, Hq, max_blocks, &G);
+    if (rc) return rc;
+    if (S == 0) return KV_OK;
+    if (!q || !out || !dev_table || !dev_ctx_lens || !aligned16(q) || !aligned16(out)) return KV_ERR_INVALID_ARG;
+    if (p->sm_count <= 0) return KV_ERR_CUDA;
+    const kv_layout &L = p->desc.layouts[layout];
+    const int variant = pick_variant(p, G);
+    kvp::AttnArgs a{};
+    a.q = q;
+    a.out = out;
+    a.table = dev_table;
+    a.ctx_lens = dev_ctx_lens;
+    a.err = p->desc.device_error;
+    a.rows_per_page = (int64_t)(p->page_bytes / (2ull * L.head_dim));
+    a.pool_pages = p->n_pages;
+    a.pages_per_block = p->pages_per_block[layout];
+    a.max_blocks = max_blocks;
+    a.S = S;
+    a.Hkv = L.num_kv_heads;
+    a.bs = p->desc.block_size;
+    a.qk_scale = scale * 1.4426950408889634f;
+    int P = 0;
+    rc = dispatch(variant, L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, false, &P);
+    if (rc) return rc;
+    size_t part_off;
+    const size_t need = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &part_off);
+    if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
+    a.ws_cnt = reinterpret_cast<int32_t *>(workspace);
+    a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
+    rc = ensure_tmap(p, layout);
+    if (rc) return rc;
+    return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
+                    true, &P);
+}
+
+}  // extern "C"

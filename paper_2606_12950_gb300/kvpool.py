@@ -1,0 +1,248 @@
+"""Thin Python binding of libkvpool's C ABI (include/kvpool.h).
+
+Argument marshalling only: every function has the C name and forwards to the
+library; device buffers are passed as raw addresses (ints) or as objects with
+``data_ptr()`` (torch tensors), streams as raw handles or objects with
+``cuda_stream``.  There is no fallback: if libkvpool.so is missing or fails to
+load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+KV_OK = 0
+KV_ERR_INVALID_ARG = -1
+KV_ERR_OUT_OF_BLOCKS = -2
+KV_ERR_CUDA = -3
+KV_ERR_DEVICE_BOUNDS = -4
+KV_ERR_UNSUPPORTED = -5
+KV_ERR_WORKSPACE = -6
+KV_ERR_DEVICE_TIMEOUT = -7
+KV_MAX_LAYOUTS = 4
+
+_NAMES = {
+    0: "KV_OK", -1: "KV_ERR_INVALID_ARG", -2: "KV_ERR_OUT_OF_BLOCKS", -3: "KV_ERR_CUDA",
+    -4: "KV_ERR_DEVICE_BOUNDS", -5: "KV_ERR_UNSUPPORTED", -6: "KV_ERR_WORKSPACE",
+    -7: "KV_ERR_DEVICE_TIMEOUT",
+}
+
+
+class KVError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} failed: {_NAMES.get(code, code)}")
+        self.code = code
+
+
+class kv_layout(ctypes.Structure):
+    _fields_ = [("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32)]
+
+
+class kv_pool_desc(ctypes.Structure):
+    _fields_ = [
+        ("device_base", ctypes.c_void_p),
+        ("pool_bytes", ctypes.c_uint64),
+        ("block_size", ctypes.c_int32),
+        ("num_layouts", ctypes.c_int32),
+        ("layouts", kv_layout * KV_MAX_LAYOUTS),
+        ("page_bytes", ctypes.c_uint64),
+        ("device_error", ctypes.c_void_p),
+        ("shuffle_seed", ctypes.c_uint64),
+    ]
+
+
+class kv_stats(ctypes.Structure):
+    _fields_ = [
+        ("pages_total", ctypes.c_int64),
+        ("pages_unassigned", ctypes.c_int64),
+        ("blocks_used", ctypes.c_int64 * KV_MAX_LAYOUTS),
+        ("blocks_cached", ctypes.c_int64 * KV_MAX_LAYOUTS),
+        ("blocks_capacity", ctypes.c_int64 * KV_MAX_LAYOUTS),
+        ("bytes_used", ctypes.c_uint64),
+        ("bytes_total", ctypes.c_uint64),
+    ]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libkvpool.so (building it first if its sources are newer)."""
+    global _lib
+    if _lib is None:
+        path = _build.LIB
+        if _build.needs_build():
+            path = _build.build()
+        if not os.path.exists(path):
+            raise RuntimeError("libkvpool.so is not built; run paper_2606_12950_gb300.build.build()")
+        L = ctypes.CDLL(path)
+        P, I, I32, I64, U64, F, SZ = (ctypes.c_void_p, ctypes.c_int, ctypes.c_int32, ctypes.c_int64,
+                                       ctypes.c_uint64, ctypes.c_float, ctypes.c_size_t)
+        sigs = {
+            "kv_pool_create": [ctypes.POINTER(kv_pool_desc), ctypes.POINTER(P)],
+            "kv_pool_destroy": [P],
+            "kv_alloc_blocks": [P, I, I, P],
+            "kv_free_blocks": [P, I, I, P],
+            "kv_block_ref": [P, I, I, P],
+            "kv_block_refcount": [P, I32, ctypes.POINTER(I32)],
+            "kv_pool_stats": [P, ctypes.POINTER(kv_stats)],
+            "kv_pool_get_error": [P, P, P],
+            "kv_block_table_upload": [P, I, P, I, I, P, P, P, P],
+            "kv_append": [P, I, P, P, P, P, I, I, P],
+            "kv_workspace_bytes": [P, I, I, I, I, I, ctypes.POINTER(SZ)],
+            "kv_workspace_clear": [P, SZ, P],
+            "paged_decode_attn": [P, I, P, P, P, P, I, I, I, F, I, P, SZ, P],
+            "kv_set_attn_variant": [P, I],
+        }
+        for name, args in sigs.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = ctypes.c_int
+        L.kv_version.argtypes = []
+        L.kv_version.restype = ctypes.c_char_p
+        _lib = L
+    return _lib
+
+
+def _addr(x) -> int | None:
+    if x is None:
+        return None
+    if hasattr(x, "data_ptr"):
+        return int(x.data_ptr())
+    return int(x)
+
+
+def _stream(s) -> int | None:
+    if s is None:
+        return None
+    if hasattr(s, "cuda_stream"):
+        return int(s.cuda_stream)
+    return int(s)
+
+
+def _check(fn: str, rc: int) -> None:
+    if rc != KV_OK:
+        raise KVError(fn, rc)
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def kv_version() -> str:
+    return lib().kv_version().decode()
+
+
+def kv_pool_create(device_base, pool_bytes: int, block_size: int, layouts, device_error,
+                   page_bytes: int = 0, shuffle_seed: int = 0) -> int:
+    """Return an opaque pool handle.  ``layouts`` is a list of (Hkv, d)."""
+    d = kv_pool_desc()
+    d.device_base = _addr(device_base)
+    d.pool_bytes = int(pool_bytes)
+    d.block_size = int(block_size)
+    d.num_layouts = len(layouts)
+    for i, (hkv, hd) in enumerate(layouts):
+        d.layouts[i] = kv_layout(int(hkv), int(hd))
+    d.page_bytes = int(page_bytes)
+    d.device_error = _addr(device_error)
+    d.shuffle_seed = int(shuffle_seed)
+    h = ctypes.c_void_p()
+    _check("kv_pool_create", lib().kv_pool_create(ctypes.byref(d), ctypes.byref(h)))
+    return h.value
+
+
+def kv_pool_destroy(pool) -> None:
+    _check("kv_pool_destroy", lib().kv_pool_destroy(pool))
+
+
+def kv_alloc_blocks(pool, layout: int, n: int) -> np.ndarray:
+    out = np.empty(max(0, int(n)), dtype=np.int32)
+    _check("kv_alloc_blocks", lib().kv_alloc_blocks(pool, layout, int(n), out.ctypes.data))
+    return out
+
+
+def kv_free_blocks(pool, layout: int, ids) -> None:
+    ids = _i32(ids)
+    _check("kv_free_blocks", lib().kv_free_blocks(pool, layout, int(ids.size), ids.ctypes.data))
+
+
+def kv_block_ref(pool, layout: int, ids) -> None:
+    ids = _i32(ids)
+    _check("kv_block_ref", lib().kv_block_ref(pool, layout, int(ids.size), ids.ctypes.data))
+
+
+def kv_block_refcount(pool, block_id: int) -> int:
+    c = ctypes.c_int32()
+    _check("kv_block_refcount", lib().kv_block_refcount(pool, int(block_id), ctypes.byref(c)))
+    return int(c.value)
+
+
+def kv_pool_stats(pool) -> dict:
+    s = kv_stats()
+    _check("kv_pool_stats", lib().kv_pool_stats(pool, ctypes.byref(s)))
+    return {
+        "pages_total": s.pages_total, "pages_unassigned": s.pages_unassigned,
+        "blocks_used": list(s.blocks_used), "blocks_cached": list(s.blocks_cached),
+        "blocks_capacity": list(s.blocks_capacity), "bytes_used": s.bytes_used,
+        "bytes_total": s.bytes_total,
+    }
+
+
+def kv_pool_get_error(pool, stream, host_buf=None) -> int:
+    """Read-and-clear the device error word; synchronises ``stream``'s work
+    up to this point when ``host_buf`` (a pinned int32 host tensor) is None."""
+    if host_buf is None:
+        code = ctypes.c_int32(0)
+        _check("kv_pool_get_error", lib().kv_pool_get_error(pool, _stream(stream), ctypes.addressof(code)))
+        import torch
+
+        torch.cuda.synchronize()
+        return int(code.value)
+    _check("kv_pool_get_error", lib().kv_pool_get_error(pool, _stream(stream), _addr(host_buf)))
+    return 0
+
+
+def kv_block_table_upload(pool, layout: int, host_table, host_ctx_lens, dev_table, dev_ctx_lens,
+                          stream=None) -> None:
+    t = host_table if isinstance(host_table, np.ndarray) and host_table.dtype == np.int32 \
+        and host_table.flags.c_contiguous else _i32(host_table)
+    lens = _i32(host_ctx_lens)
+    S, max_blocks = t.shape
+    _check("kv_block_table_upload",
+           lib().kv_block_table_upload(pool, layout, t.ctypes.data, int(S), int(max_blocks),
+                                       lens.ctypes.data, _addr(dev_table), _addr(dev_ctx_lens),
+                                       _stream(stream)))
+
+
+def kv_append(pool, layout: int, k_new, v_new, dev_table, dev_ctx_lens, max_blocks: int, S: int,
+              stream=None) -> None:
+    _check("kv_append", lib().kv_append(pool, layout, _addr(k_new), _addr(v_new), _addr(dev_table),
+                                        _addr(dev_ctx_lens), int(max_blocks), int(S), _stream(stream)))
+
+
+def kv_workspace_bytes(pool, layout: int, S: int, Hq: int, max_blocks: int, num_splits: int = 0) -> int:
+    n = ctypes.c_size_t(0)
+    _check("kv_workspace_bytes", lib().kv_workspace_bytes(pool, layout, int(S), int(Hq), int(max_blocks),
+                                                          int(num_splits), ctypes.byref(n)))
+    return int(n.value)
+
+
+def kv_workspace_clear(workspace, ws_bytes: int, stream=None) -> None:
+    _check("kv_workspace_clear", lib().kv_workspace_clear(_addr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def paged_decode_attn(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_blocks: int, S: int,
+                      Hq: int, scale: float, num_splits: int, workspace, ws_bytes: int,
+                      stream=None) -> None:
+    _check("paged_decode_attn",
+           lib().paged_decode_attn(pool, layout, _addr(q), _addr(out), _addr(dev_table),
+                                   _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq), float(scale),
+                                   int(num_splits), _addr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def kv_set_attn_variant(pool, variant: int) -> None:
+    _check("kv_set_attn_variant", lib().kv_set_attn_variant(pool, int(variant)))

@@ -1,0 +1,116 @@
+"""Device-side holders for a pool and a decode batch, driving the C ABI.
+
+PyTorch provides the device memory and the streams; every step of the path
+(append, attention, split combine) runs in libkvpool's kernels through
+``kvpool``.  Host arrays use uint16 for bf16 bit patterns.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import kvpool as K
+
+
+def _dev_u16(a: np.ndarray, device) -> torch.Tensor:
+    """Host uint16 (bf16 bits) -> device bfloat16 tensor with the same bits."""
+    t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16))
+    return t.to(device).view(torch.bfloat16)
+
+
+def _host_u16(t: torch.Tensor) -> np.ndarray:
+    return t.view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+class DevicePool:
+    """A caller-owned device buffer managed by a kv_pool handle."""
+
+    def __init__(self, n_pages: int, page_bytes: int, block_size: int, layouts, shuffle_seed: int = 0,
+                 device: str = "cuda"):
+        self.device = torch.device(device)
+        self.n_pages = int(n_pages)
+        self.page_bytes = int(page_bytes)
+        self.buf = torch.empty(self.n_pages * self.page_bytes, dtype=torch.uint8, device=self.device)
+        self.err = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.handle = K.kv_pool_create(self.buf, self.buf.numel(), block_size, layouts, self.err,
+                                       page_bytes=page_bytes, shuffle_seed=shuffle_seed)
+
+    def upload(self, pool_u16: np.ndarray) -> None:
+        src = torch.from_numpy(np.ascontiguousarray(pool_u16).view(np.uint8))
+        self.buf.copy_(src.to(self.device))
+
+    def fill_u16(self, value: int) -> None:
+        self.buf.view(torch.int16).fill_(np.array(value, np.uint16).view(np.int16).item())
+
+    def download(self) -> np.ndarray:
+        return self.buf.cpu().numpy().view(np.uint16)
+
+    def error(self, stream=None) -> int:
+        return K.kv_pool_get_error(self.handle, stream)
+
+    def set_variant(self, v: int) -> None:
+        K.kv_set_attn_variant(self.handle, v)
+
+    def close(self) -> None:
+        if self.handle:
+            K.kv_pool_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class DeviceBatch:
+    """One layout's decode batch on the device (q, new K/V rows, table,
+    lengths, output, workspace)."""
+
+    def __init__(self, pool: DevicePool, layout: int, b, num_splits: int = 0):
+        dev = pool.device
+        self.pool = pool
+        self.layout = layout
+        self.b = b
+        self.S, self.Hq, self.d, self.max_blocks = b.S, b.Hq, b.d, b.max_blocks
+        self.q = _dev_u16(b.q, dev)
+        self.k_new = _dev_u16(b.k_new, dev)
+        self.v_new = _dev_u16(b.v_new, dev)
+        self.table = torch.empty((b.S, b.max_blocks), dtype=torch.int32, device=dev)
+        self.lens = torch.empty(b.S, dtype=torch.int32, device=dev)
+        self.out = torch.empty((b.S, b.Hq, b.d), dtype=torch.bfloat16, device=dev)
+        self.num_splits = num_splits
+        self.ws_bytes = K.kv_workspace_bytes(pool.handle, layout, b.S, b.Hq, b.max_blocks, num_splits)
+        self.ws = torch.zeros(max(256, self.ws_bytes), dtype=torch.uint8, device=dev)
+        self.upload_table(b.table, b.ctx_lens)
+
+    def upload_table(self, table, lens, stream=None) -> None:
+        K.kv_block_table_upload(self.pool.handle, self.layout, table, lens, self.table, self.lens, stream)
+
+    def set_rows(self, q, k_new, v_new) -> None:
+        dev = self.pool.device
+        self.q.copy_(_dev_u16(q, dev))
+        self.k_new.copy_(_dev_u16(k_new, dev))
+        self.v_new.copy_(_dev_u16(v_new, dev))
+
+    def append(self, stream=None) -> None:
+        K.kv_append(self.pool.handle, self.layout, self.k_new, self.v_new, self.table, self.lens,
+                    self.max_blocks, self.S, stream)
+
+    def attend(self, num_splits: int | None = None, stream=None) -> None:
+        ns = self.num_splits if num_splits is None else num_splits
+        if ns != self.num_splits:
+            need = K.kv_workspace_bytes(self.pool.handle, self.layout, self.S, self.Hq, self.max_blocks, ns)
+            if need > self.ws.numel():
+                self.ws = torch.zeros(need, dtype=torch.uint8, device=self.pool.device)
+            self.num_splits = ns
+            self.ws_bytes = need
+        K.paged_decode_attn(self.pool.handle, self.layout, self.q, self.out, self.table, self.lens,
+                            self.max_blocks, self.S, self.Hq, self.b.scale, ns, self.ws,
+                            self.ws.numel(), stream)
+
+    def out_f64(self) -> np.ndarray:
+        return self.out.float().cpu().numpy().astype(np.float64)
+
+    def out_bits(self) -> np.ndarray:
+        return _host_u16(self.out)
