@@ -567,8 +567,12 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         __syncthreads();
     }
 
+    // with fewer units than CTAs only the first W CTAs take work, so that
+    // every working CTA's range is non-empty and a run's contributors are
+    // exactly the CTAs cta_of(first unit) .. cta_of(last unit)
     const int64_t W = T[S];
-    const int64_t P = a.P;
+    const int64_t P = W < (int64_t)a.P ? W : (int64_t)a.P;
+    if ((int64_t)blockIdx.x >= P) return;
     const int32_t u0 = (int32_t)((int64_t)blockIdx.x * W / P);
     const int32_t u1 = (int32_t)((int64_t)(blockIdx.x + 1) * W / P);
     if (u0 >= u1) return;  // no units for this CTA (no barriers are shared beyond here)
