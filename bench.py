@@ -329,7 +329,7 @@ def main():
                      "peak_kind": peak_kind, "attn_ms": attn_avg_ms},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": 3 * args.steps,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,

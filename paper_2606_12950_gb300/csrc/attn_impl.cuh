@@ -10,17 +10,25 @@
 // Work decomposition (all decided on the device from the lengths):
 //   unit  = one 16-token tile of one (sequence, KV head) run; a run of n
 //           tokens has ceil(n/16) units; units are ordered (s, g, tile).
-//   CTA i of P processes the contiguous unit range [i*W/P, (i+1)*W/P): every
-//           CTA streams the same number of bytes (+-1 tile) whatever the
-//           length distribution.
-//   piece = the part of one run inside one CTA's range.  A run covered by
-//           one CTA is finished in place; a run cut by CTA boundaries leaves
-//           one fp32 partial (max, sum, unnormalised output) per CTA, and the
-//           last CTA to arrive (per-run counter) merges them in CTA order.
-// Inside a CTA each of the 4 warps owns every 4th unit of a piece and a
-// private ring of shared-memory stages fed by 2-D TMA loads (128-byte
-// swizzle) that run ahead across piece boundaries.  The 4 warps' states are
-// merged through shared memory at the end of a piece.
+//   part  = one of NP = P * 8 equal contiguous unit ranges [i*W/NP,
+//           (i+1)*W/NP), one per warp of the P resident CTAs: every warp
+//           streams the same number of bytes (+-1 tile) whatever the length
+//           distribution.
+//   piece = the part of one run inside one part.  A run covered by one part
+//           is finished in place; a run cut by part boundaries leaves one
+//           fp32 partial (max, sum, unnormalised output) per part, which the
+//           combine kernel below merges in part order.
+// Inside a CTA each of the 8 warps is one part of that split: it streams its
+// own contiguous range of units through its own shared-memory stage, issuing
+// its own 2-D TMA loads (128-byte swizzle) of each unit's K and V tiles with
+// one mbarrier for K and one for V: the next unit's K streams in while the
+// warp does softmax and P.V on the current one, the next V while it does the
+// next q.K.  (Measured on GB300: one issuing thread per SM cannot keep HBM
+// busy with these 2 KB boxes; one per warp can.)  The pool rows of the CTA's
+// units are resolved from the block table in the prologue, while the memory
+// system is idle, so no table load sits on the streaming path.  A run that
+// ends inside a warp's range is written out by that warp directly; no state
+// is merged between warps of a CTA.
 //
 // Two compute variants share this skeleton:
 //   FmaCompute : CUDA-core FFMA2 dot products and weighted sums.
@@ -41,10 +49,10 @@
 
 namespace kvp {
 
-constexpr int kWarps = 4;
+constexpr int kWarps = 8;  // each warp streams and computes its own units
 constexpr int kThreads = kWarps * 32;
-constexpr int kTile = 16;              // tokens per unit
-constexpr uint32_t kHalfBytes = kTile * 128;  // one 64-column box: 16 rows x 128 B
+constexpr int kTile = 16;                         // tokens per unit
+constexpr uint32_t kHalfBytes = kTile * 128;      // one 64-column box: 16 rows x 128 B
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
 struct AttnArgs {
@@ -54,7 +62,7 @@ struct AttnArgs {
     const int32_t *ctx_lens;
     int32_t *err;
     float *ws_part;
-    int32_t *ws_cnt;
+    int32_t *ws_T;           // T[0..S] and NP, for the combine kernel
     int64_t rows_per_page;   // page_bytes / (d * 2)
     int64_t pool_pages;
     int32_t pages_per_block;
@@ -62,7 +70,7 @@ struct AttnArgs {
     int32_t S;
     int32_t Hkv;
     int32_t bs;
-    int32_t nsw;             // stages per warp
+    int32_t rows_cap;        // units whose pool rows are resolved up front
     int32_t P;               // CTAs (work partitions)
     float qk_scale;          // scale * log2(e)
 };
@@ -71,7 +79,7 @@ __device__ __forceinline__ void report(int32_t *err, int code) { atomicCAS(err, 
 
 // bounded wait on an mbarrier phase; a wait that exceeds the limit records
 // KV_ERR_DEVICE_TIMEOUT and makes every later wait of this warp return at once
-__device__ __forceinline__ void wait_stage(uint32_t bar, uint32_t parity, int32_t *err, bool &dead)
+__device__ __forceinline__ void wait_phase(uint32_t bar, uint32_t parity, int32_t *err, bool &dead)
 {
     if (dead) return;
     if (mbar_try_wait(bar, parity)) return;
@@ -99,6 +107,7 @@ __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 
 // ------------------------------------------------------------ CUDA cores ---
 template <int D, int G>
 struct FmaCompute {
+    static constexpr int kMinBlocks = 1;                     // registers allow one CTA per SM
     static constexpr int LPT = (G * D / 8 <= 64) ? 8 : 16;  // lanes per token
     static constexpr int EPL = D / LPT;                      // elements per lane
     static constexpr int NCH = EPL / 8;                      // 16-byte chunks per lane
@@ -110,7 +119,8 @@ struct FmaCompute {
     float2 o[G][EPL / 2];
     float m[G];
     float l[G];
-    int grp, sub;
+    float p[TPG][G];
+    int grp, sub, nv;
 
     __device__ __forceinline__ void begin(const uint16_t *qrow, float qk_scale, int lane)
     {
@@ -134,8 +144,10 @@ struct FmaCompute {
         }
     }
 
-    __device__ __forceinline__ void tile(const uint8_t *Ks, const uint8_t *Vs, int nvalid)
+    // q.K for the tile's tokens, online-softmax update, weights p
+    __device__ __forceinline__ void qk(const uint8_t *Ks, int nvalid)
     {
+        nv = nvalid;
         float sc[TPG][G];
 #pragma unroll
         for (int i = 0; i < TPG; ++i) {
@@ -196,13 +208,18 @@ struct FmaCompute {
         for (int i = 0; i < TPG; ++i)
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                sc[i][h] = fast_exp2(sc[i][h] - m[h]);
-                l[h] += sc[i][h];
+                p[i][h] = fast_exp2(sc[i][h] - m[h]);
+                l[h] += p[i][h];
             }
+    }
+
+    // o += p * V for the tile's valid tokens
+    __device__ __forceinline__ void pv(uint8_t *Vs)
+    {
 #pragma unroll
         for (int i = 0; i < TPG; ++i) {
             const int t = grp + i * NGRP;
-            if (t < nvalid) {
+            if (t < nv) {
 #pragma unroll
                 for (int j = 0; j < NCH; ++j) {
                     uint4 w = *reinterpret_cast<const uint4 *>(Vs + swz(t, sub + j * LPT));
@@ -212,15 +229,16 @@ struct FmaCompute {
                         float2 vv = make_float2(bf_lo(ws[e]), bf_hi(ws[e]));
 #pragma unroll
                         for (int h = 0; h < G; ++h)
-                            o[h][j * 4 + e] = __ffma2_rn(make_float2(sc[i][h], sc[i][h]), vv, o[h][j * 4 + e]);
+                            o[h][j * 4 + e] = __ffma2_rn(make_float2(p[i][h], p[i][h]), vv, o[h][j * 4 + e]);
                     }
                 }
             }
         }
     }
 
-    // write this warp's (o[G][D], m[G], l[G]) to shared memory
-    __device__ __forceinline__ void finish(float *mw, int lane)
+    // end of a piece: the bf16 output o / l (whole run in this warp), or the
+    // fp32 partial (o unnormalised, m, l) of this warp's part of the run
+    __device__ __forceinline__ void store(uint16_t *orow, float *slot, bool split, int lane)
     {
 #pragma unroll
         for (int off = LPT; off < 32; off <<= 1)
@@ -239,16 +257,27 @@ struct FmaCompute {
 #pragma unroll
                 for (int j = 0; j < NCH; ++j) {
                     const int c = sub + j * LPT;
-                    float4 *dst = reinterpret_cast<float4 *>(mw + h * D + c * 8);
-                    dst[0] = make_float4(o[h][j * 4 + 0].x, o[h][j * 4 + 0].y, o[h][j * 4 + 1].x, o[h][j * 4 + 1].y);
-                    dst[1] = make_float4(o[h][j * 4 + 2].x, o[h][j * 4 + 2].y, o[h][j * 4 + 3].x, o[h][j * 4 + 3].y);
+                    if (!split) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            __nv_bfloat162 b2 =
+                                __floats2bfloat162_rn(o[h][j * 4 + e].x / l[h], o[h][j * 4 + e].y / l[h]);
+                            w[e] = *reinterpret_cast<uint32_t *>(&b2);
+                        }
+                        *reinterpret_cast<uint4 *>(orow + h * D + c * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+                    } else {
+                        float4 *dst = reinterpret_cast<float4 *>(slot + h * D + c * 8);
+                        dst[0] = make_float4(o[h][j * 4 + 0].x, o[h][j * 4 + 0].y, o[h][j * 4 + 1].x, o[h][j * 4 + 1].y);
+                        dst[1] = make_float4(o[h][j * 4 + 2].x, o[h][j * 4 + 2].y, o[h][j * 4 + 3].x, o[h][j * 4 + 3].y);
+                    }
                 }
         }
-        if (lane == 0) {
+        if (split && lane == 0) {
 #pragma unroll
             for (int h = 0; h < G; ++h) {
-                mw[G * D + h] = m[h];
-                mw[G * D + G + h] = l[h];
+                slot[G * D + h] = m[h];
+                slot[G * D + G + h] = l[h];
             }
         }
     }
@@ -258,12 +287,14 @@ struct FmaCompute {
 template <int D, int G>
 struct MmaCompute {
     static_assert(G <= 8, "query-head group must fit the n=8 MMA tile");
+    static constexpr int kMinBlocks = 2;
     static constexpr int KS = D / 16;
     uint32_t qf[KS][2];  // B operand of q.K: Q^T fragments (bf16x2)
     float acc[KS][4];    // O^T accumulators, 16 d-rows per block
     float m[2], l[2];    // heads 2*tig, 2*tig+1
+    uint32_t pb0, pb1;   // B operand of P.V (P^T fragments)
     float qk_scale;
-    int gid, tig, lane_;
+    int gid, tig, lane_, nv;
 
     __device__ __forceinline__ void begin(const uint16_t *qrow, float scale, int lane)
     {
@@ -287,21 +318,10 @@ struct MmaCompute {
         l[0] = l[1] = 0.f;
     }
 
-    __device__ __forceinline__ void tile(const uint8_t *Ks, uint8_t *Vs, int nvalid)
+    __device__ __forceinline__ void qk(const uint8_t *Ks, int nvalid)
     {
-        // rows past the context may hold anything (even NaN bit patterns);
-        // P is zero there, but 0 * NaN is NaN inside the MMA, so clear them
-        if (nvalid < kTile) {
-            const int nchunk = (kTile - nvalid) * (D / 8);
-            for (int idx = lane_; idx < nchunk; idx += 32) {
-                const int r = nvalid + idx / (D / 8);
-                const int c = idx % (D / 8);
-                *reinterpret_cast<uint4 *>(Vs + swz(r, c)) = make_uint4(0u, 0u, 0u, 0u);
-            }
-            __syncwarp();
-        }
+        nv = nvalid;
         const uint32_t kbase = smem_u32(Ks);
-        const uint32_t vbase = smem_u32(Vs);
         const int mat = lane_ >> 3, r8 = lane_ & 7;
         float s[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
@@ -312,16 +332,17 @@ struct MmaCompute {
         }
         // s[0], s[1]: token gid, heads 2tig, 2tig+1; s[2], s[3]: token gid+8
         const bool ok0 = gid < nvalid, ok1 = gid + 8 < nvalid;
-        float x0 = ok0 ? s[0] * qk_scale : -INFINITY;
-        float x1 = ok0 ? s[1] * qk_scale : -INFINITY;
-        float x2 = ok1 ? s[2] * qk_scale : -INFINITY;
-        float x3 = ok1 ? s[3] * qk_scale : -INFINITY;
+        const float x0 = ok0 ? s[0] * qk_scale : -INFINITY;
+        const float x1 = ok0 ? s[1] * qk_scale : -INFINITY;
+        const float x2 = ok1 ? s[2] * qk_scale : -INFINITY;
+        const float x3 = ok1 ? s[3] * qk_scale : -INFINITY;
         float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3);
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
             t0 = fmaxf(t0, __shfl_xor_sync(0xffffffffu, t0, off));
             t1 = fmaxf(t1, __shfl_xor_sync(0xffffffffu, t1, off));
         }
+        // lazy rescale (see FmaCompute::qk)
         if (t0 > m[0] + 8.f) {
             const float a = fast_exp2(m[0] - t0);
             l[0] *= a;
@@ -348,17 +369,35 @@ struct MmaCompute {
         l[1] += p1 + p3;
         __nv_bfloat162 lo = __floats2bfloat162_rn(p0, p1);
         __nv_bfloat162 hi = __floats2bfloat162_rn(p2, p3);
-        const uint32_t b0 = movmatrix_trans(*reinterpret_cast<uint32_t *>(&lo));
-        const uint32_t b1 = movmatrix_trans(*reinterpret_cast<uint32_t *>(&hi));
+        pb0 = movmatrix_trans(*reinterpret_cast<uint32_t *>(&lo));
+        pb1 = movmatrix_trans(*reinterpret_cast<uint32_t *>(&hi));
+    }
+
+    __device__ __forceinline__ void pv(uint8_t *Vs)
+    {
+        // rows past the context may hold anything (even NaN bit patterns);
+        // P is zero there, but 0 * NaN is NaN inside the MMA, so clear them
+        if (nv < kTile) {
+            const int nchunk = (kTile - nv) * (D / 8);
+            for (int idx = lane_; idx < nchunk; idx += 32) {
+                const int r = nv + idx / (D / 8);
+                const int c = idx % (D / 8);
+                *reinterpret_cast<uint4 *>(Vs + swz(r, c)) = make_uint4(0u, 0u, 0u, 0u);
+            }
+            __syncwarp();
+        }
+        const uint32_t vbase = smem_u32(Vs);
+        const int mat = lane_ >> 3, r8 = lane_ & 7;
 #pragma unroll
         for (int mb = 0; mb < KS; ++mb) {
             uint32_t a0, a1, a2, a3;
             ldmatrix_x4_trans(vbase + swz(r8 + (mat >> 1) * 8, mb * 2 + (mat & 1)), a0, a1, a2, a3);
-            mma_bf16_16816(acc[mb], a0, a1, a2, a3, b0, b1);
+            mma_bf16_16816(acc[mb], a0, a1, a2, a3, pb0, pb1);
         }
     }
 
-    __device__ __forceinline__ void finish(float *mw, int lane)
+    // end of a piece (see FmaCompute::store)
+    __device__ __forceinline__ void store(uint16_t *orow, float *slot, bool split, int lane)
     {
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
@@ -366,35 +405,48 @@ struct MmaCompute {
             l[1] += __shfl_xor_sync(0xffffffffu, l[1], off);
         }
         const int h0 = 2 * tig, h1 = 2 * tig + 1;
+        if (!split) {
 #pragma unroll
-        for (int mb = 0; mb < KS; ++mb) {
-            const int d0 = mb * 16 + gid;
-            if (h0 < G) {
-                mw[h0 * D + d0] = acc[mb][0];
-                mw[h0 * D + d0 + 8] = acc[mb][2];
+            for (int mb = 0; mb < KS; ++mb) {
+                const int d0 = mb * 16 + gid;
+                if (h0 < G) {
+                    orow[h0 * D + d0] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[mb][0] / l[0]));
+                    orow[h0 * D + d0 + 8] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[mb][2] / l[0]));
+                }
+                if (h1 < G) {
+                    orow[h1 * D + d0] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[mb][1] / l[1]));
+                    orow[h1 * D + d0 + 8] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[mb][3] / l[1]));
+                }
             }
-            if (h1 < G) {
-                mw[h1 * D + d0] = acc[mb][1];
-                mw[h1 * D + d0 + 8] = acc[mb][3];
+        } else {
+#pragma unroll
+            for (int mb = 0; mb < KS; ++mb) {
+                const int d0 = mb * 16 + gid;
+                if (h0 < G) {
+                    slot[h0 * D + d0] = acc[mb][0];
+                    slot[h0 * D + d0 + 8] = acc[mb][2];
+                }
+                if (h1 < G) {
+                    slot[h1 * D + d0] = acc[mb][1];
+                    slot[h1 * D + d0 + 8] = acc[mb][3];
+                }
             }
-        }
-        if (gid == 0) {
-            if (h0 < G) {
-                mw[G * D + h0] = m[0];
-                mw[G * D + G + h0] = l[0];
-            }
-            if (h1 < G) {
-                mw[G * D + h1] = m[1];
-                mw[G * D + G + h1] = l[1];
+            if (gid == 0) {
+                if (h0 < G) {
+                    slot[G * D + h0] = m[0];
+                    slot[G * D + G + h0] = l[0];
+                }
+                if (h1 < G) {
+                    slot[G * D + h1] = m[1];
+                    slot[G * D + G + h1] = l[1];
+                }
             }
         }
         (void)lane;
     }
 };
 
-// ---------------------------------------------------------------- stream ---
-// Walks one warp's units across the pieces of its CTA's range: within a piece
-// [pb, pe) the warp owns units pb + warp, pb + warp + 4, ...
+// ----------------------------------------------------------- work units ---
 struct Piece {
     int32_t pb, pe;        // piece unit range
     int32_t run_begin;     // unit id of tile 0 of this (s, g) run
@@ -413,15 +465,21 @@ __device__ __forceinline__ int32_t clamp_len(const AttnArgs &a, int s, bool repo
     return n;
 }
 
-// T[s] = first unit of sequence s (T[S] = total); find the run holding u
-__device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T, int32_t u, int32_t u1, Piece &p)
+// largest s with T[s] <= u; T[s] = first unit of sequence s, T[S] = total,
+// so empty sequences (T[s] == T[s+1]) are skipped
+__device__ __forceinline__ int find_seq(const int32_t *T, int S, int32_t u)
 {
-    int lo = 0, hi = a.S;  // largest s with T[s] <= u (T is non-decreasing)
+    int lo = 0, hi = S;
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
         if (T[mid] <= u) lo = mid; else hi = mid;
     }
-    const int s = lo;
+    return lo;
+}
+
+__device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T, int32_t u, int32_t u1, Piece &p)
+{
+    const int s = find_seq(T, a.S, u);
     const int32_t nt = (T[s + 1] - T[s]) / a.Hkv;
     const int32_t g = (u - T[s]) / nt;
     p.s = s;
@@ -433,78 +491,54 @@ __device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T
     p.pe = p.run_end < u1 ? p.run_end : u1;
 }
 
-struct Producer {
-    Piece p;
-    int32_t u;   // next unit to load
-    int32_t u1;
-    bool valid;
-
-    __device__ __forceinline__ void normalise(const AttnArgs &a, const int32_t *T, int warp)
-    {
-        while (valid && u >= p.pe) {
-            if (p.pe >= u1) {
-                valid = false;
-                break;
-            }
-            decode_piece(a, T, p.pe, u1, p);
-            u = p.pb + warp;
-        }
-    }
-    __device__ __forceinline__ void start(const AttnArgs &a, const int32_t *T, int32_t u0, int32_t uend, int warp)
-    {
-        u1 = uend;
-        valid = u0 < uend;
-        if (!valid) return;
-        decode_piece(a, T, u0, u1, p);
-        u = p.pb + warp;
-        normalise(a, T, warp);
-    }
-    __device__ __forceinline__ void advance(const AttnArgs &a, const int32_t *T, int warp)
-    {
-        u += kWarps;
-        normalise(a, T, warp);
-    }
-};
-
-template <int D>
-__device__ __forceinline__ void issue_unit(const CUtensorMap *tmap, const AttnArgs &a, const Producer &pr,
-                                           uint32_t stage_addr, uint32_t bar, uint64_t policy)
+// Pool row of unit u's K tile (TMA y coordinate; V is Hkv*bs rows further),
+// or -1 if the block table names a block outside the pool.
+__device__ __forceinline__ int32_t unit_row(const AttnArgs &a, const int32_t *T, int32_t u)
 {
-    constexpr int HALVES = D / 64;
-    constexpr uint32_t TILE_BYTES = HALVES * kHalfBytes;
-    const int32_t tile = pr.u - pr.p.run_begin;
-    const int32_t tok0 = tile * kTile;
-    const int32_t lb = tok0 / a.bs;
-    const int32_t phys = a.table[(int64_t)pr.p.s * a.max_blocks + lb];
-    if (phys < 0 || (int64_t)phys + a.pages_per_block > a.pool_pages) {
-        report(a.err, KV_ERR_DEVICE_BOUNDS);
-        mbar_arrive(bar);  // complete the phase without data
-        return;
-    }
-    const int64_t row0 = (int64_t)phys * a.rows_per_page + (tok0 % a.bs);
-    const int32_t yk = (int32_t)(row0 + (int64_t)pr.p.g * a.bs);
-    const int32_t yv = (int32_t)(row0 + (int64_t)(a.Hkv + pr.p.g) * a.bs);
-    mbar_arrive_expect_tx(bar, 2 * TILE_BYTES);
-#pragma unroll
-    for (int h = 0; h < HALVES; ++h) {
-        tma_load_2d(stage_addr + h * kHalfBytes, tmap, h * 64, yk, bar, policy);
-        tma_load_2d(stage_addr + TILE_BYTES + h * kHalfBytes, tmap, h * 64, yv, bar, policy);
-    }
+    const int s = find_seq(T, a.S, u);
+    const int32_t nt = (T[s + 1] - T[s]) / a.Hkv;
+    const int32_t within = u - T[s];
+    const int32_t g = within / nt;
+    const int32_t tok0 = (within - g * nt) * kTile;
+    const int32_t phys = a.table[(int64_t)s * a.max_blocks + tok0 / a.bs];
+    if (phys < 0 || (int64_t)phys + a.pages_per_block > a.pool_pages) return -1;
+    return (int32_t)((int64_t)phys * a.rows_per_page + (tok0 % a.bs) + (int64_t)g * a.bs);
 }
 
-// first CTA whose range contains unit u
+// the part (of NP) whose range contains unit u
 __device__ __forceinline__ int32_t cta_of(int64_t u, int64_t W, int64_t P)
 {
     return (int32_t)(((u + 1) * P - 1) / W);
 }
 
-// per-warp merge record and per-CTA partial: o[G][D], m[G], l[G], padded to
-// a multiple of 4 floats so every record starts 16-byte aligned
+// per-part partial: o[G][D], m[G], l[G], padded to a multiple of 4 floats so
+// every record starts 16-byte aligned
 template <int D, int G>
 __host__ __device__ constexpr uint32_t merge_floats() { return (G * D + 2 * G + 3) / 4 * 4; }
 
+// Load K (which = 0) or V (which = 1) of unit u into this warp's stage;
+// completes on `bar`.  Lane 0 only.
+template <int D>
+__device__ __forceinline__ void issue_half(const CUtensorMap *tmap, const AttnArgs &a, const int32_t *T,
+                                           const int32_t *rows, int32_t cu0, int32_t u, int which, uint32_t dst,
+                                           uint32_t bar, uint64_t policy)
+{
+    constexpr int HALVES = D / 64;
+    const int32_t k = u - cu0;
+    int32_t y = k < a.rows_cap ? rows[k] : unit_row(a, T, u);
+    if (y < 0) {
+        report(a.err, KV_ERR_DEVICE_BOUNDS);
+        mbar_arrive(bar);  // complete the phase without data
+        return;
+    }
+    y += which * a.Hkv * a.bs;
+    mbar_arrive_expect_tx(bar, HALVES * kHalfBytes);
+#pragma unroll
+    for (int h = 0; h < HALVES; ++h) tma_load_2d(dst + h * kHalfBytes, tmap, h * 64, y, bar, policy);
+}
+
 template <int D, int G, class Comp>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, Comp::kMinBlocks)
 paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ AttnArgs a)
 {
     constexpr int HALVES = D / 64;
@@ -514,23 +548,22 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     extern __shared__ uint8_t smem_raw[];
     // stages need 1024-byte alignment for the 128-byte swizzle pattern
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-    const int nsw = a.nsw;
-    uint8_t *stages = smem;
-    float *merge = reinterpret_cast<float *>(smem + (size_t)kWarps * nsw * STAGE_BYTES);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(merge + kWarps * MF);
-    int32_t *misc = reinterpret_cast<int32_t *>(bars + kWarps * nsw);  // [0..7] scratch
-    int32_t *T = misc + 8;                                              // [S + 1]
+    uint8_t *stages = smem;                                                              // [kWarps][STAGE]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kWarps * STAGE_BYTES);  // K[w], V[w]
+    int32_t *misc = reinterpret_cast<int32_t *>(bars + 2 * kWarps);                     // [16] scratch
+    int32_t *T = misc + 16;                                                              // [S + 1]
+    int32_t *rows = T + a.S + 1;                                                         // [rows_cap]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int S = a.S, Hkv = a.Hkv, Hq = a.Hkv * G;
 
     if (tid == 0) {
-        for (int i = 0; i < kWarps * nsw; ++i) mbar_init(smem_u32(&bars[i]), 1);
+        for (int i = 0; i < 2 * kWarps; ++i) mbar_init(smem_u32(&bars[i]), 1);
         fence_mbar_init();
     }
     if (tid == 32) prefetch_tensormap(&tmap);
 
-    // ---- prologue: T[s] = first unit of sequence s ----
+    // ---- prologue 1: T[s] = first unit of sequence s ----
     {
         const int per = (S + kThreads - 1) / kThreads;
         const int lo = min(S, tid * per), hi = min(S, lo + per);
@@ -543,7 +576,6 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
                 for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
             }
         }
-        // block exclusive scan of `local`
         int32_t incl = local;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
@@ -567,25 +599,44 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         __syncthreads();
     }
 
-    // with fewer units than CTAs only the first W CTAs take work, so that
-    // every working CTA's range is non-empty and a run's contributors are
-    // exactly the CTAs cta_of(first unit) .. cta_of(last unit)
+    // The W units are cut into NP = min(P * kWarps, W) equal parts; part i is
+    // [i*W/NP, (i+1)*W/NP) and belongs to warp i % kWarps of CTA i / kWarps.
+    // With NP <= W every part is non-empty, so a run's contributors are
+    // exactly the parts part_of(first unit) .. part_of(last unit).
     const int64_t W = T[S];
-    const int64_t P = W < (int64_t)a.P ? W : (int64_t)a.P;
-    if ((int64_t)blockIdx.x >= P) return;
-    const int32_t u0 = (int32_t)((int64_t)blockIdx.x * W / P);
-    const int32_t u1 = (int32_t)((int64_t)(blockIdx.x + 1) * W / P);
-    if (u0 >= u1) return;  // no units for this CTA (no barriers are shared beyond here)
+    const int64_t NP = W < (int64_t)a.P * kWarps ? W : (int64_t)a.P * kWarps;
+    if (blockIdx.x == 0) {  // the combine kernel needs the same split
+        for (int i = tid; i <= S; i += kThreads) a.ws_T[i] = T[i];
+        if (tid == 0) a.ws_T[S + 1] = (int32_t)NP;
+    }
+    const int64_t first_part = (int64_t)blockIdx.x * kWarps;
+    if (first_part >= NP) return;
+    const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
+    const int32_t cu0 = (int32_t)(first_part * W / NP);                             // this CTA's units
+    const int32_t cu1 = (int32_t)(last_part * W / NP);
+
+    // ---- prologue 2: resolve the block table for this CTA's units while the
+    // memory system is idle (later lookups would queue behind the TMA stream)
+    {
+        const int32_t nr = min(cu1 - cu0, a.rows_cap);
+        for (int32_t k = tid; k < nr; k += kThreads) rows[k] = unit_row(a, T, cu0 + k);
+        __syncthreads();
+    }
+
+    const int64_t part = first_part + warp;
+    if (part >= NP) return;  // no CTA-wide barrier below this point
+    const int32_t u0 = (int32_t)(part * W / NP);
+    const int32_t u1 = (int32_t)((part + 1) * W / NP);
 
     const uint64_t policy = l2_policy_evict_first();
-    uint8_t *my_stages = stages + (size_t)warp * nsw * STAGE_BYTES;
-    uint64_t *my_bars = bars + warp * nsw;
+    uint8_t *Ks = stages + (size_t)warp * STAGE_BYTES;
+    uint8_t *Vs = Ks + TILE_BYTES;
+    const uint32_t k_addr = smem_u32(Ks), v_addr = smem_u32(Vs);
+    const uint32_t bk = smem_u32(&bars[warp]), bv = smem_u32(&bars[kWarps + warp]);
 
-    Producer pr;
-    pr.start(a, T, u0, u1, warp);
-    for (int k = 0; k < nsw && pr.valid; ++k) {
-        if (lane == 0) issue_unit<D>(&tmap, a, pr, smem_u32(my_stages + k * STAGE_BYTES), smem_u32(&my_bars[k]), policy);
-        pr.advance(a, T, warp);
+    if (lane == 0) {
+        issue_half<D>(&tmap, a, T, rows, cu0, u0, 0, k_addr, bk, policy);
+        issue_half<D>(&tmap, a, T, rows, cu0, u0, 1, v_addr, bv, policy);
     }
 
     bool dead = false;
@@ -596,98 +647,161 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         decode_piece(a, T, u, u1, pc);
         Comp comp;
         comp.begin(a.q + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D, a.qk_scale, lane);
-        for (int32_t uu = pc.pb + warp; uu < pc.pe; uu += kWarps) {
-            const uint32_t st = consumed % (uint32_t)nsw;
-            wait_stage(smem_u32(&my_bars[st]), (consumed / (uint32_t)nsw) & 1u, a.err, dead);
-            uint8_t *Ks = my_stages + st * STAGE_BYTES;
-            const int32_t tok0 = (uu - pc.run_begin) * kTile;
-            const int nvalid = min(kTile, pc.n - tok0);
-            comp.tile(Ks, Ks + TILE_BYTES, nvalid);
-            // this stage is refilled by TMA next: order the warp's generic
-            // shared-memory accesses before the async-proxy write
+        for (int32_t uu = pc.pb; uu < pc.pe; ++uu) {
+            const uint32_t par = consumed & 1u;
+            const int nvalid = min(kTile, pc.n - (uu - pc.run_begin) * kTile);
+            const bool more = uu + 1 < u1;
+            wait_phase(bk, par, a.err, dead);
+            comp.qk(Ks, nvalid);
+            // the K stage is refilled by TMA next: order the warp's generic
+            // shared-memory reads before the async-proxy write
             fence_proxy_async_smem();
             __syncwarp();
-            if (pr.valid) {
-                if (lane == 0) {
-                    issue_unit<D>(&tmap, a, pr, smem_u32(Ks), smem_u32(&my_bars[st]), policy);
-                }
-                pr.advance(a, T, warp);
-            }
+            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 0, k_addr, bk, policy);
+            wait_phase(bv, par, a.err, dead);
+            comp.pv(Vs);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 1, v_addr, bv, policy);
             ++consumed;
         }
-        comp.finish(merge + warp * MF, lane);
-        __syncthreads();
 
-        // ---- merge the 4 warps; finish the run or leave a partial ----
+        // ---- end of a piece: the output, or this part's partial ----
         const int32_t r = pc.s * Hkv + pc.g;
-        const int32_t i_first = cta_of(pc.run_begin, W, P);
-        const int32_t i_last = cta_of(pc.run_end - 1, W, P);
-        const bool split = i_first != i_last;
-        float *slot = a.ws_part + (int64_t)(r + (int32_t)blockIdx.x) * MF;
+        const int32_t p_first = cta_of(pc.run_begin, W, NP);
+        const int32_t p_last = cta_of(pc.run_end - 1, W, NP);
+        const bool split = p_first != p_last;
         uint16_t *orow = a.out + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D;
-        for (int idx = tid; idx < G * D; idx += kThreads) {
-            const int h = idx / D;
-            float M = -INFINITY;
-#pragma unroll
-            for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge[w * MF + G * D + h]);
-            float L = 0.f, O = 0.f;
-#pragma unroll
-            for (int w = 0; w < kWarps; ++w) {
-                const float sc = fast_exp2(merge[w * MF + G * D + h] - M);
-                L += sc * merge[w * MF + G * D + G + h];
-                O += sc * merge[w * MF + idx];
-            }
-            if (!split) {
-                orow[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(O / L));
-            } else {
-                slot[idx] = O;
-                if (idx % D == 0) {
-                    slot[G * D + h] = M;
-                    slot[G * D + G + h] = L;
-                }
-            }
-        }
-        if (split) {
-            __threadfence();
-            __syncthreads();
-            if (tid == 0) {
-                const int32_t prev = atomicAdd(&a.ws_cnt[r], 1);
-                const int last = prev == i_last - i_first;
-                if (last) atomicExch(&a.ws_cnt[r], 0);
-                misc[4] = last;
-            }
-            __syncthreads();
-            if (misc[4]) {
-                __threadfence();
-                const float *base = a.ws_part + (int64_t)(r + i_first) * MF;
-                const int cnt = i_last - i_first + 1;
-                for (int idx = tid; idx < G * D; idx += kThreads) {
-                    const int h = idx / D;
-                    float M = -INFINITY;
-                    for (int k = 0; k < cnt; ++k) M = fmaxf(M, __ldcg(base + (int64_t)k * MF + G * D + h));
-                    float L = 0.f, O = 0.f;
-                    for (int k = 0; k < cnt; ++k) {
-                        const float *sl = base + (int64_t)k * MF;
-                        const float sc = fast_exp2(__ldcg(sl + G * D + h) - M);
-                        L += sc * __ldcg(sl + G * D + G + h);
-                        O += sc * __ldcg(sl + idx);
-                    }
-                    orow[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(O / L));
-                }
-            }
-        }
-        __syncthreads();
+        float *slot = a.ws_part + ((int64_t)r + part) * MF;
+        comp.store(orow, slot, split, lane);
         u = pc.pe;
     }
 }
 
-// host helpers ---------------------------------------------------------------
+// ------------------------------------------------------------ combine ---
+// Split-K combine: for each (sequence, KV head) run cut by part boundaries,
+// merge its parts' partials (m_k, l_k, o_k) in part order:
+//     M = max_k m_k,  out = sum_k 2^(m_k - M) o_k / sum_k 2^(m_k - M) l_k
+// (base-2 online-softmax state).  One CTA per run; runs finished inside the
+// attention kernel return at once.
+constexpr int kCombineThreads = 256;
+
+struct CombineArgs {
+    uint16_t *out;
+    const int32_t *ws_T;   // T[0..S], NP
+    const float *ws_part;
+    int32_t S;
+    int32_t Hkv;
+};
+
+// columns (float4 of o) per combine CTA, and CTAs per run
 template <int D, int G>
-inline size_t attn_smem_bytes(int nsw, int S)
+__host__ __device__ constexpr int combine_cols()
+{
+    return G * D / 4 < 32 ? G * D / 4 : ((G * D / 4) % 32 == 0 ? 32 : 16);
+}
+template <int D, int G>
+__host__ __device__ constexpr int combine_ctas_per_run() { return (G * D / 4) / combine_cols<D, G>(); }
+
+template <int D, int G>
+__global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_constant__ CombineArgs c)
+{
+    constexpr uint32_t MF = merge_floats<D, G>();
+    constexpr int CW = combine_cols<D, G>();       // columns of this CTA
+    constexpr int CB = combine_ctas_per_run<D, G>();
+    constexpr int NSPLIT = kCombineThreads / CW;   // thread groups splitting the partials
+    static_assert(CW * CB == G * D / 4, "columns must tile the output");
+    __shared__ float s_max[kCombineThreads / 32][G];
+    __shared__ float s_M[G];
+    __shared__ float4 s_O[kCombineThreads];
+    __shared__ float s_L[kCombineThreads];
+    const int r = blockIdx.x / CB, cb = blockIdx.x % CB;
+    const int s = r / c.Hkv, g = r % c.Hkv;
+    const int64_t W = c.ws_T[c.S], NP = c.ws_T[c.S + 1];
+    if (W == 0) return;
+    const int32_t nt = (c.ws_T[s + 1] - c.ws_T[s]) / c.Hkv;
+    if (nt == 0) return;
+    const int64_t run_begin = c.ws_T[s] + (int64_t)g * nt;
+    const int32_t p_first = cta_of(run_begin, W, NP);
+    const int32_t p_last = cta_of(run_begin + nt - 1, W, NP);
+    if (p_first == p_last) return;
+    const int cnt = p_last - p_first + 1;
+    const float *base = c.ws_part + ((int64_t)r + p_first) * MF;
+    uint16_t *orow = c.out + ((int64_t)s * c.Hkv * G + (int64_t)g * G) * D;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // M_h = max over the partials, all (partial, head) pairs in parallel
+    float mx[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
+    for (int k = tid; k < cnt; k += kCombineThreads)
+#pragma unroll
+        for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], base[(int64_t)k * MF + G * D + h]);
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], off));
+        if (lane == 0) s_max[warp][h] = mx[h];
+    }
+    __syncthreads();
+    if (tid < G) {
+        float M = -INFINITY;
+        for (int w = 0; w < kCombineThreads / 32; ++w) M = fmaxf(M, s_max[w][tid]);
+        s_M[tid] = M;
+    }
+    __syncthreads();
+
+    // weighted sums: thread (group, column) takes partials group, group + NSPLIT, ...
+    const int col = cb * CW + tid % CW;
+    const int grp = tid / CW;
+    const int h = (col * 4) / D;
+    const float M = s_M[h];
+    float L = 0.f;
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int k = grp; k < cnt; k += NSPLIT) {
+        const float *sl = base + (int64_t)k * MF;
+        const float sc = fast_exp2(sl[G * D + h] - M);
+        L += sc * sl[G * D + G + h];
+        const float4 o = *reinterpret_cast<const float4 *>(sl + col * 4);
+        O.x += sc * o.x;
+        O.y += sc * o.y;
+        O.z += sc * o.z;
+        O.w += sc * o.w;
+    }
+    s_O[tid] = O;
+    s_L[tid] = L;
+    __syncthreads();
+    if (grp == 0) {
+        // groups in order, so the sum order depends only on the run's shape
+        for (int j = 1; j < NSPLIT; ++j) {
+            const float4 o = s_O[tid + j * CW];
+            O.x += o.x;
+            O.y += o.y;
+            O.z += o.z;
+            O.w += o.w;
+            L += s_L[tid + j * CW];
+        }
+        __nv_bfloat162 lo = __floats2bfloat162_rn(O.x / L, O.y / L);
+        __nv_bfloat162 hi = __floats2bfloat162_rn(O.z / L, O.w / L);
+        uint2 w2;
+        w2.x = *reinterpret_cast<uint32_t *>(&lo);
+        w2.y = *reinterpret_cast<uint32_t *>(&hi);
+        *reinterpret_cast<uint2 *>(orow + col * 4) = w2;
+    }
+}
+
+// host helpers ---------------------------------------------------------------
+constexpr int kRowsCap = 2048;
+
+template <int D, int G>
+inline size_t attn_smem_bytes(int S, int rows_cap)
 {
     const size_t stage = 2ull * (D / 64) * kHalfBytes;
-    return 1024 + (size_t)kWarps * nsw * stage + (size_t)kWarps * merge_floats<D, G>() * 4 +
-           (size_t)kWarps * nsw * 8 + 32 + (size_t)(S + 1) * 4;
+    return 1024 + (size_t)kWarps * stage + (2 * kWarps) * 8 + 64 + (size_t)(S + 1) * 4 + (size_t)rows_cap * 4;
 }
+
+// partial records: one per (run, part) pair that a run can touch
+inline size_t attn_partial_slots(int S, int Hkv, int P) { return (size_t)S * Hkv + (size_t)P * kWarps; }
 
 }  // namespace kvp

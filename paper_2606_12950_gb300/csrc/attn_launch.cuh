@@ -10,8 +10,9 @@
 
 namespace kvp {
 
-// shared memory a CTA may use so that two CTAs fit on one SM
-constexpr size_t kSmemBudget = 113 * 1024;
+// shared memory of one CTA: up to 227 KB; the block-table window (rows of the
+// CTA's units resolved in the prologue) is kRowsCap entries
+constexpr size_t kSmemMax = 227 * 1024;
 
 template <int D, int G, class Comp>
 int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaStream_t st, bool launch,
@@ -20,24 +21,23 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     auto fn = paged_attn_kernel<D, G, Comp>;
     static std::atomic<bool> attr_set{false};
     if (!attr_set.load()) {
-        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024) != cudaSuccess)
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMax) != cudaSuccess)
             return KV_ERR_CUDA;
         attr_set.store(true);
     }
-    const size_t stage = 2ull * (D / 64) * kHalfBytes;
-    const size_t fixed = attn_smem_bytes<D, G>(0, a.S);
-    int nsw = 2;
-    if (fixed < kSmemBudget) nsw = (int)std::min<size_t>(6, std::max<size_t>(2, (kSmemBudget - fixed) / (kWarps * stage)));
-    const size_t smem = attn_smem_bytes<D, G>(nsw, a.S);
-    if (smem > 227 * 1024) return KV_ERR_INVALID_ARG;
+    const size_t smem = attn_smem_bytes<D, G>(a.S, kRowsCap);
+    if (smem > kSmemMax) return KV_ERR_INVALID_ARG;  // S too large for the per-CTA sequence index
     int occ = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, kThreads, smem) != cudaSuccess) return KV_ERR_CUDA;
     const int P = P_req > 0 ? P_req : std::max(1, occ) * std::max(1, sm_count);
     *P_out = P;
     if (!launch) return KV_OK;
-    a.nsw = nsw;
+    a.rows_cap = kRowsCap;
     a.P = P;
     fn<<<P, kThreads, smem, st>>>(*tmap, a);
+    if (cudaGetLastError() != cudaSuccess) return KV_ERR_CUDA;
+    CombineArgs c{a.out, a.ws_T, a.ws_part, a.S, a.Hkv};
+    combine_kernel<D, G><<<a.S * a.Hkv * combine_ctas_per_run<D, G>(), kCombineThreads, 0, st>>>(c);
     return cudaGetLastError() == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 

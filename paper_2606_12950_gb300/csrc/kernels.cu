@@ -122,11 +122,12 @@ int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::Attn
     return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, launch, P_out);
 }
 
+// workspace: T[0..S] and NP (int32, padded to 256 bytes), then the partials
 size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
 {
-    const size_t cnt = ((size_t)S * Hkv * 4 + 255) / 256 * 256;
-    *part_off = cnt;
-    return cnt + ((size_t)S * Hkv + (size_t)P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
+    const size_t hdr = ((size_t)(S + 2) * 4 + 255) / 256 * 256;
+    *part_off = hdr;
+    return hdr + kvp::attn_partial_slots(S, Hkv, P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
 
 }  // namespace
@@ -205,7 +206,7 @@ int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, 
     size_t part_off;
     const size_t need = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &part_off);
     if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
-    a.ws_cnt = reinterpret_cast<int32_t *>(workspace);
+    a.ws_T = reinterpret_cast<int32_t *>(workspace);
     a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
