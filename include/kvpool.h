@@ -227,6 +227,32 @@ int paged_decode_attn(kv_pool *pool, int layout, const uint16_t *q, uint16_t *ou
                       size_t ws_bytes, void *stream);
 
 /*
+ * paged_decode_attn for callers that cannot allocate device memory.  The
+ * paper has no counterpart; this is a service of this library.  Callers that
+ * cannot hand over a workspace include a server whose KV pool already holds
+ * all free HBM, a host framework whose allocator this layer may not call,
+ * and a decode loop in which a cudaMalloc (which may synchronise the whole
+ * device) is not acceptable.
+ * Arguments and results are those of paged_decode_attn without the
+ * workspace.  The split-K scratch is instead a fixed 32 MiB device array
+ * inside the library, which every GPU that loads the library holds until
+ * the process exits.  The call allocates nothing.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - If kv_workspace_bytes for the same arguments exceeds 32 MiB the call
+ *     returns KV_ERR_WORKSPACE and launches nothing; use paged_decode_attn
+ *     with a workspace for such batches.
+ *   - Every call uses the same array, which keeps the last call's contents.
+ *     Nothing in it has to start at zero (each call writes what it reads),
+ *     but calls that can overlap on the GPU (streams with no ordering
+ *     between them) race on it; calls on one stream are ordered.
+ */
+int paged_decode_attn_noalloc(kv_pool *pool, int layout, const uint16_t *q, uint16_t *out,
+                              const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks,
+                              int S, int Hq, float scale, int num_splits, void *stream);
+
+/*
  * Select the attention compute variant for later calls on this pool:
  * 0 = automatic (the fastest measured for the shape), 1 = CUDA-core FMA,
  * 2 = warp-level tensor-core MMA (mma.sync bf16, fp32 accumulate).

@@ -96,6 +96,7 @@ def lib() -> ctypes.CDLL:
             "kv_workspace_bytes": [P, I, I, I, I, I, ctypes.POINTER(SZ)],
             "kv_workspace_clear": [P, SZ, P],
             "paged_decode_attn": [P, I, P, P, P, P, I, I, I, F, I, P, SZ, P],
+            "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
             "kv_set_attn_variant": [P, I],
         }
         for name, args in sigs.items():
@@ -242,6 +243,16 @@ def paged_decode_attn(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_bl
            lib().paged_decode_attn(pool, layout, _addr(q), _addr(out), _addr(dev_table),
                                    _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq), float(scale),
                                    int(num_splits), _addr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_blocks: int, S: int,
+                              Hq: int, scale: float, num_splits: int = 0, stream=None) -> None:
+    """paged_decode_attn with the library's fixed 32 MiB scratch instead of a
+    caller workspace (for callers that cannot allocate)."""
+    _check("paged_decode_attn_noalloc",
+           lib().paged_decode_attn_noalloc(pool, layout, _addr(q), _addr(out), _addr(dev_table),
+                                           _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq), float(scale),
+                                           int(num_splits), _stream(stream)))
 
 
 def kv_set_attn_variant(pool, variant: int) -> None:
