@@ -3,9 +3,11 @@
 layer (64 sequences, 32 query / 8 KV heads, head dim 128, block size 16,
 lognormal context lengths with median 1024, sigma 1, clipped to 16384).
 
-A step is the whole hot path for one batch: upload of the step's context
-lengths (with the block table), append of every sequence's new K/V row, and
-paged decode attention (with its in-kernel split combine).  The headline
+A step is the whole hot path for one batch: the host sequence table advances
+every sequence by one token (growing reservations where needed) and syncs the
+lengths and changed table entries to the device, then the new K/V rows are
+appended and paged decode attention runs (attention kernel + split-K
+combine).  The headline
 value is algorithmic HBM GB/s of the step: K/V bytes read (each sequence's
 whole context) + q read + output written + appended K/V written, divided by
 the device time of the step.
@@ -205,31 +207,44 @@ def main():
     from paper_2606_12950_gb300 import workloads as W
     from paper_2606_12950_gb300.runner import DeviceBatch, DevicePool
 
-    b = W.config2_llama8b(steps=max(100, args.steps + args.warmup + 2))
-    pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)])
+    total_steps = 2 * (args.warmup + args.steps) + 8
+    b = W.config2_llama8b(steps=max(100, total_steps))
+    pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)], shuffle_seed=b.meta["seed"])
     pool.upload(b.pool)
     if args.variant:
         pool.set_variant(args.variant)
     db = DeviceBatch(pool, 0, b, args.num_splits)
     stream = torch.cuda.current_stream()
 
-    # pinned host copies of the table and lengths (uploaded every step)
-    table_h = torch.from_numpy(b.table.copy()).pin_memory()
-    lens0 = b.ctx_lens.astype(np.int32)
-    nsteps = args.warmup + args.steps
-    lens_h = [torch.from_numpy(lens0 + i).pin_memory() for i in range(nsteps)]
+    # host sequence table: each sequence reserves its whole run up front
+    # (Eq. 2 with the true total length); blocks come from the shuffled pool
+    seqtab = K.SeqTab(pool.handle, 0, b.S, b.max_blocks)
+    pre = b.meta["pre_lens"].astype(np.int64)
+    for s in range(b.S):
+        seqtab.reserve(s, int(pre[s]) + total_steps)
+        seqtab.set_len(s, int(pre[s]))
+    done = [0]  # decode steps issued so far
 
-    def step(i, ev_pair=None):
-        K.kv_block_table_upload(pool.handle, 0, table_h.numpy(), lens_h[i].numpy(), db.table, db.lens, stream)
+    def step_bytes(j):
+        """algorithmic bytes of decode step j: (attention call, whole step)"""
+        n = pre + 1 + j
+        kv = int(n.sum()) * 2 * b.Hkv * b.d * 2
+        qo = 2 * b.S * b.Hq * b.d * 2
+        return kv + qo, kv + qo + 2 * b.S * b.Hkv * b.d * 2
+
+    def step(ev_pair=None):
+        seqtab.advance()                         # host: every live sequence gains this step's token
+        seqtab.sync(db.table, db.lens, stream)   # lengths (and any changed entries) to the device
         db.append(stream)
         if ev_pair is not None:
             ev_pair[0].record(stream)
         db.attend(stream=stream)
         if ev_pair is not None:
             ev_pair[1].record(stream)
+        done[0] += 1
 
     for i in range(args.warmup):
-        step(i)
+        step()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
@@ -242,9 +257,10 @@ def main():
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
+    first = done[0]
     t_start.record(stream)
     for i in range(args.steps):
-        step(args.warmup + i, evs[i])
+        step(evs[i])
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -256,15 +272,8 @@ def main():
         ms = float(tt.item())
     err = pool.error(stream)
 
-    # algorithmic bytes over the timed steps (lengths grow by one per step)
-    kv_total = 0
-    attn_bytes = []
-    for i in range(args.steps):
-        n = lens0.astype(np.int64) + args.warmup + i
-        kv = int(n.sum()) * 2 * b.Hkv * b.d * 2
-        qo = 2 * b.S * b.Hq * b.d * 2
-        kv_total += kv + qo + 2 * b.S * b.Hkv * b.d * 2
-        attn_bytes.append(kv + qo)
+    attn_bytes = [step_bytes(first + i)[0] for i in range(args.steps)]
+    kv_total = sum(step_bytes(first + i)[1] for i in range(args.steps))
     gbs = kv_total / (ms * 1e-3) / 1e9 * world
     tokens_per_s = b.S * args.steps / (ms * 1e-3) * world
     attn_avg_ms = float(np.mean(attn_ms))
@@ -274,29 +283,30 @@ def main():
     # end to end: q / k / v from pinned host memory, output back to host
     q_h = [torch.from_numpy(x.view(np.int16)).pin_memory() for x in W_step_rows(b, 0)]
     out_h = torch.empty(db.out.shape, dtype=torch.bfloat16).pin_memory()
-    h2d = sum(int(t.numel()) * 2 for t in q_h) + table_h.numel() * 4 + b.S * 4
+    h2d = sum(int(t.numel()) * 2 for t in q_h) + b.S * 4
     d2h = out_h.numel() * 2
 
-    def e2e_step(i):
+    def e2e_step():
         db.q.view(torch.int16).copy_(q_h[0], non_blocking=True)
         db.k_new.view(torch.int16).copy_(q_h[1], non_blocking=True)
         db.v_new.view(torch.int16).copy_(q_h[2], non_blocking=True)
-        step(i)
+        step()
         out_h.copy_(db.out, non_blocking=True)
 
-    # restore the lengths so the e2e pass replays the same steps
     for i in range(3):
-        e2e_step(i)
+        e2e_step()
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+    first_e2e = done[0]
     e0.record(stream)
     for i in range(args.steps):
-        e2e_step(args.warmup + i)
+        e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
+    e2e_total = sum(step_bytes(first_e2e + i)[1] for i in range(args.steps))
     e2e_ms = e0.elapsed_time(e1)
-    e2e_gbs = kv_total / (e2e_ms * 1e-3) / 1e9 * world
+    e2e_gbs = e2e_total / (e2e_ms * 1e-3) / 1e9 * world
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -319,7 +329,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": WORKLOAD, "S": b.S, "Hq": b.Hq, "Hkv": b.Hkv, "d": b.d, "bs": b.bs,
-                   "context_tokens_first_step": int(lens0.sum()) + args.warmup,
+                   "context_tokens_first_step": int((pre + 1 + first).sum()),
                    "kv_bytes_per_step": int(attn_bytes[0]), "l2": "inputs larger than L2 (no flush needed)",
                    "num_splits": args.num_splits, "variant": args.variant,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
@@ -329,7 +339,7 @@ def main():
                      "peak_kind": peak_kind, "attn_ms": attn_avg_ms},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": 4 * args.steps,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,

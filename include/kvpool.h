@@ -176,6 +176,88 @@ int kv_block_table_upload(kv_pool *pool, int layout, const int32_t *host_table, 
                           int max_blocks, const int32_t *host_ctx_lens, int32_t *dev_table,
                           int32_t *dev_ctx_lens, void *stream);
 
+/* ------------------------------------------------------ sequence tables --- */
+
+/*
+ * A host sequence table of one layout: for each of max_seqs slots, its block
+ * list (the row of the block table) and its post-append length.  It carries
+ * the runtime's side of the paper's per-stage KV provisioning: a stage
+ * reserves ceil((P + L^)/bs) blocks for its predicted total length (Eq. 2),
+ * a prediction that falls short grows the reservation one block at a time
+ * (a "reservation miss"), a shared prompt prefix is held by reference, and
+ * blocks go back to the pool when a stage or sequence ends (§III-C).  Every
+ * change is recorded so that kv_seqtab_sync sends only changed table entries
+ * to the device.  Not thread-safe; one table per host thread.
+ */
+typedef struct kv_seqtab kv_seqtab;
+
+typedef struct kv_seqtab_counters {
+    int64_t blocks_held;        /* block references held by all rows */
+    int64_t reserve_calls;
+    int64_t reservation_misses; /* one-block growths in kv_seq_advance */
+    int64_t releases;
+    int64_t entries_uploaded;   /* table entries sent by kv_seqtab_sync */
+    int64_t sync_launches;
+} kv_seqtab_counters;
+
+/* Create an empty table (all lengths 0, all entries -1).  KV_ERR_INVALID_ARG. */
+int kv_seqtab_create(kv_pool *pool, int layout, int max_seqs, int max_blocks, kv_seqtab **out);
+
+/* Release every block reference the table holds, then the table. */
+int kv_seqtab_destroy(kv_seqtab *t);
+
+/*
+ * Make slot s hold at least ceil(tokens / bs) blocks (Eq. 2's reservation
+ * for a stage of P + L^ tokens), allocating the missing ones from the pool.
+ * All-or-nothing: KV_ERR_OUT_OF_BLOCKS leaves the slot unchanged; more than
+ * max_blocks is KV_ERR_INVALID_ARG.
+ */
+int kv_seq_reserve(kv_seqtab *t, int s, int64_t tokens);
+
+/*
+ * Give the empty slot dst the first nblocks blocks of slot src by reference
+ * (refcount + 1 each), e.g. a system prompt shared by every agent of a
+ * workflow.  The shared blocks must be full (dst's own tokens start at
+ * nblocks * bs).  KV_ERR_INVALID_ARG if dst is not empty or src holds fewer.
+ */
+int kv_seq_share_prefix(kv_seqtab *t, int dst, int src, int nblocks);
+
+/* Set slot s's length (0 .. held blocks * bs).  KV_ERR_INVALID_ARG. */
+int kv_seq_set_len(kv_seqtab *t, int s, int32_t len);
+
+/*
+ * One decode step for n slots (seqs == NULL: every slot with length > 0):
+ * length += 1; a slot whose held blocks are full first grows by one block
+ * (a reservation miss).  All-or-nothing over the call: if the pool cannot
+ * supply every needed block, KV_ERR_OUT_OF_BLOCKS and nothing changes.
+ * *n_grown (may be NULL) receives the number of slots that grew.
+ */
+int kv_seq_advance(kv_seqtab *t, int n, const int32_t *seqs, int32_t *n_grown);
+
+/* Drop every block reference of slot s and set its length to 0. */
+int kv_seq_release(kv_seqtab *t, int s);
+
+/* Drop slot s's reserved blocks beyond ceil(length / bs) (end of a stage). */
+int kv_seq_trim(kv_seqtab *t, int s);
+
+/*
+ * Bring a device copy of the table up to date on `stream`: every slot's
+ * length goes to dev_ctx_lens[0 .. max_seqs), and every table entry changed
+ * since the previous sync (of this table, to any device copy) goes to
+ * dev_table (int32 [max_seqs][max_blocks]).  The values travel as kernel
+ * parameters, so the host table may change right after the call returns.
+ * The first sync after create sends the whole table.
+ */
+int kv_seqtab_sync(kv_seqtab *t, int32_t *dev_table, int32_t *dev_ctx_lens, void *stream);
+
+/*
+ * Read-only host views: table int32 [max_seqs][max_blocks] (-1 = no block)
+ * and lengths int32 [max_seqs]; valid until the next call that changes t.
+ */
+int kv_seqtab_host(const kv_seqtab *t, const int32_t **table, const int32_t **ctx_lens);
+
+int kv_seqtab_get_counters(const kv_seqtab *t, kv_seqtab_counters *out);
+
 /* -------------------------------------------------------------- kernels --- */
 
 /*
@@ -192,15 +274,16 @@ int kv_append(kv_pool *pool, int layout, const uint16_t *k_new, const uint16_t *
 
 /*
  * Bytes of device workspace paged_decode_attn needs for these sizes and this
- * num_splits.  The workspace holds per-(sequence, KV head) arrival counters
- * followed by fp32 split partials; its counter area must be zero before the
- * first call that uses it (allocate it zero-filled, or call
- * kv_workspace_clear once); every call that completes leaves it zero again.
+ * num_splits: the batch's split index (S + 2 int32) followed by fp32 split
+ * partials, one record of G*d + 2*G floats per (sequence, KV head, part)
+ * pair a split run can produce.  Every call writes all it reads, so the
+ * workspace needs no initialisation and may be reused freely by calls that
+ * are ordered on one stream.
  */
 int kv_workspace_bytes(const kv_pool *pool, int layout, int S, int Hq, int max_blocks,
                        int num_splits, size_t *out_bytes);
 
-/* Zero a workspace on `stream` (cudaMemsetAsync). */
+/* Zero a workspace on `stream` (cudaMemsetAsync); not required before use. */
 int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream);
 
 /*
@@ -212,14 +295,15 @@ int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream);
  * q, out: bf16 [S][Hq][d] device arrays.  A sequence with n == 0 gets zeros.
  * Arithmetic: fp32 products and accumulation, online softmax in base 2,
  * bf16 output rounded to nearest-even.
- * Work split: the KV range of each sequence is cut into chunks of whole
- * blocks; num_splits == 0 picks one chunk size for the batch from the SM
- * count and the total length; num_splits > 0 cuts every sequence into at
- * most num_splits equal block-aligned chunks.  Chunk partials (max, sum,
- * unnormalised output) are combined in fixed chunk order, so results do not
- * depend on where blocks sit in the pool.
+ * Work split: the batch's KV is cut into 16-token tiles of one (sequence,
+ * KV head); the tiles are split into equal contiguous parts, one per warp of
+ * the resident CTAs (num_splits == 0), or into num_splits * 8 parts when
+ * num_splits > 0 CTAs are requested.  A (sequence, head) whose tiles fall in
+ * more than one part leaves fp32 partials (max, sum, unnormalised output)
+ * that a second kernel merges in part order, so results do not depend on
+ * where blocks sit in the pool.  Launches two kernels on `stream`.
  * Errors: KV_ERR_INVALID_ARG, KV_ERR_UNSUPPORTED (d not 64/128, G not in
- * {1,2,3,4,5,6,8}), KV_ERR_WORKSPACE.
+ * {1,2,4,5,8}, block size not a multiple of 16), KV_ERR_WORKSPACE.
  */
 int paged_decode_attn(kv_pool *pool, int layout, const uint16_t *q, uint16_t *out,
                       const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks,

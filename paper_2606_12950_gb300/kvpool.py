@@ -55,6 +55,17 @@ class kv_pool_desc(ctypes.Structure):
     ]
 
 
+class kv_seqtab_counters(ctypes.Structure):
+    _fields_ = [
+        ("blocks_held", ctypes.c_int64),
+        ("reserve_calls", ctypes.c_int64),
+        ("reservation_misses", ctypes.c_int64),
+        ("releases", ctypes.c_int64),
+        ("entries_uploaded", ctypes.c_int64),
+        ("sync_launches", ctypes.c_int64),
+    ]
+
+
 class kv_stats(ctypes.Structure):
     _fields_ = [
         ("pages_total", ctypes.c_int64),
@@ -98,6 +109,17 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn": [P, I, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
             "kv_set_attn_variant": [P, I],
+            "kv_seqtab_create": [P, I, I, I, ctypes.POINTER(P)],
+            "kv_seqtab_destroy": [P],
+            "kv_seq_reserve": [P, I, I64],
+            "kv_seq_share_prefix": [P, I, I, I],
+            "kv_seq_set_len": [P, I, I32],
+            "kv_seq_advance": [P, I, P, ctypes.POINTER(I32)],
+            "kv_seq_release": [P, I],
+            "kv_seq_trim": [P, I],
+            "kv_seqtab_sync": [P, P, P, P],
+            "kv_seqtab_host": [P, ctypes.POINTER(P), ctypes.POINTER(P)],
+            "kv_seqtab_get_counters": [P, ctypes.POINTER(kv_seqtab_counters)],
         }
         for name, args in sigs.items():
             f = getattr(L, name)
@@ -257,3 +279,69 @@ def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens
 
 def kv_set_attn_variant(pool, variant: int) -> None:
     _check("kv_set_attn_variant", lib().kv_set_attn_variant(pool, int(variant)))
+
+
+# ------------------------------------------------------------ sequence tables
+class SeqTab:
+    """Handle of a host sequence table (kv_seqtab_*)."""
+
+    def __init__(self, pool, layout: int, max_seqs: int, max_blocks: int):
+        h = ctypes.c_void_p()
+        _check("kv_seqtab_create", lib().kv_seqtab_create(pool, layout, int(max_seqs), int(max_blocks),
+                                                          ctypes.byref(h)))
+        self.handle = h.value
+        self.S = int(max_seqs)
+        self.max_blocks = int(max_blocks)
+
+    def close(self) -> None:
+        if self.handle:
+            _check("kv_seqtab_destroy", lib().kv_seqtab_destroy(self.handle))
+            self.handle = None
+
+    def reserve(self, s: int, tokens: int) -> None:
+        _check("kv_seq_reserve", lib().kv_seq_reserve(self.handle, int(s), int(tokens)))
+
+    def share_prefix(self, dst: int, src: int, nblocks: int) -> None:
+        _check("kv_seq_share_prefix", lib().kv_seq_share_prefix(self.handle, int(dst), int(src), int(nblocks)))
+
+    def set_len(self, s: int, length: int) -> None:
+        _check("kv_seq_set_len", lib().kv_seq_set_len(self.handle, int(s), int(length)))
+
+    def advance(self, seqs=None) -> int:
+        g = ctypes.c_int32(0)
+        if seqs is None:
+            _check("kv_seq_advance", lib().kv_seq_advance(self.handle, 0, None, ctypes.byref(g)))
+        else:
+            a = _i32(seqs)
+            _check("kv_seq_advance", lib().kv_seq_advance(self.handle, int(a.size), a.ctypes.data, ctypes.byref(g)))
+        return int(g.value)
+
+    def release(self, s: int) -> None:
+        _check("kv_seq_release", lib().kv_seq_release(self.handle, int(s)))
+
+    def trim(self, s: int) -> None:
+        _check("kv_seq_trim", lib().kv_seq_trim(self.handle, int(s)))
+
+    def sync(self, dev_table, dev_ctx_lens, stream=None) -> None:
+        _check("kv_seqtab_sync", lib().kv_seqtab_sync(self.handle, _addr(dev_table), _addr(dev_ctx_lens),
+                                                      _stream(stream)))
+
+    def host(self):
+        """Copies of the host table [S, max_blocks] and lengths [S]."""
+        t = ctypes.c_void_p()
+        l = ctypes.c_void_p()
+        _check("kv_seqtab_host", lib().kv_seqtab_host(self.handle, ctypes.byref(t), ctypes.byref(l)))
+        tab = np.ctypeslib.as_array(ctypes.cast(t, ctypes.POINTER(ctypes.c_int32)), shape=(self.S * self.max_blocks,))
+        lens = np.ctypeslib.as_array(ctypes.cast(l, ctypes.POINTER(ctypes.c_int32)), shape=(self.S,))
+        return tab.reshape(self.S, self.max_blocks).copy(), lens.copy()
+
+    def counters(self) -> dict:
+        c = kv_seqtab_counters()
+        _check("kv_seqtab_get_counters", lib().kv_seqtab_get_counters(self.handle, ctypes.byref(c)))
+        return {f: getattr(c, f) for f, _ in kv_seqtab_counters._fields_}
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
