@@ -67,11 +67,17 @@ def _c(a, dtype):
 
 
 def append(pool: np.ndarray, n_pages: int, page_elems: int, bs: int, Hkv: int, d: int,
-           k_new, v_new, table, ctx_lens) -> np.ndarray:
-    """Return a copy of ``pool`` with each sequence's new K/V row written at
-    position ctx_len-1 (bit copy)."""
+           k_new, v_new, table, ctx_lens, inplace: bool = False) -> np.ndarray:
+    """Return ``pool`` with each sequence's new K/V row written at position
+    ctx_len-1 (bit copy); a copy unless ``inplace`` (then ``pool`` must be a
+    contiguous uint16 array and is modified)."""
     lib = _load()
-    out = np.array(pool, dtype=np.uint16, copy=True)
+    if inplace:
+        if pool.dtype != np.uint16 or not pool.flags.c_contiguous:
+            raise ValueError("in-place append needs a contiguous uint16 pool")
+        out = pool
+    else:
+        out = np.array(pool, dtype=np.uint16, copy=True)
     table = _c(table, np.int32)
     ctx = _c(ctx_lens, np.int32)
     k_new = _c(k_new, np.uint16)

@@ -238,3 +238,99 @@ def step_rows(seed: int, step: int, S: int, Hq: int, Hkv: int, d: int):
     rng = np.random.default_rng([seed, 1, step])
     return (bf16_normal(rng, (S, Hq, d)), bf16_normal(rng, (S, Hkv, d)),
             bf16_normal(rng, (S, Hkv, d)))
+
+
+# ---------------------------------------------------------------------------
+# config 3: Planner -> Coder -> Reviewer agent chains
+# ---------------------------------------------------------------------------
+PREFIX_TOKENS = 2048  # system prompt shared by reference by every chain
+CHAIN_STAGES = 3
+
+
+@dataclass
+class ChainDraws:
+    """Random draws of one agent chain: the user prompt length, and per stage
+    the true output length and the factor U[0.8, 1.5] that turns it into the
+    predicted length the stage reserves for."""
+
+    prompt: int
+    out_len: np.ndarray  # int64 [CHAIN_STAGES]
+    u: np.ndarray        # float64 [CHAIN_STAGES]
+
+
+def chain_draws(rng: np.random.Generator, median: float = 300.0, sigma: float = 1.0,
+                max_out: int = 4096) -> ChainDraws:
+    prompt = int(lognormal_lengths(rng, 1, median, sigma, 1, max_out)[0])
+    out_len = lognormal_lengths(rng, CHAIN_STAGES, median, sigma, 1, max_out)
+    u = rng.uniform(0.8, 1.5, size=CHAIN_STAGES)
+    return ChainDraws(prompt, out_len, u)
+
+
+# ---------------------------------------------------------------------------
+# config 4: three co-located models in one pool filled to 90%
+# ---------------------------------------------------------------------------
+COLOC_LAYOUTS = [(32, 32), (32, 8), (40, 8)]  # (Hq, Hkv), d = 128, bs = 16
+COLOC_SPLIT = (205, 205, 102)
+
+
+def config4_colocation(seed: int = 1004, fill_pool: bool = True, fill: float = 0.9):
+    """Three layer shapes (MHA 32/32, GQA 32/8, GQA 40/8; d = 128, bs = 16)
+    sharing one pool of 64 KiB pages; an MHA block spans 4 pages.  512
+    sequences split 205/205/102 with bounded-Pareto(1.5) cached lengths on
+    [128, 32768].  The pool holds the blocks the batch needs (after this
+    step's append) plus free room so that it is `fill` full; blocks sit at
+    seeded random places.  Returns (list of Batch sharing `pool`, n_pages,
+    page_elems)."""
+    rng = np.random.default_rng(seed)
+    d, bs = 128, 16
+    page_elems = 2 * 8 * bs * d  # 64 KiB of bf16
+    lens = [bounded_pareto_lengths(rng, n, 1.5, 128, 32768) for n in COLOC_SPLIT]
+    kpages = [2 * hkv * bs * d // page_elems for _, hkv in COLOC_LAYOUTS]  # 4, 1, 1
+    nblk = [(l + 1 + bs - 1) // bs for l in lens]  # post-append
+    need_pages = sum(int(nb.sum()) * k for nb, k in zip(nblk, kpages))
+    n_super = -(-int(np.ceil(need_pages / fill)) // 4)
+    n_pages = n_super * 4
+    supers = rng.permutation(n_super)
+    # MHA blocks take whole superpages; GQA blocks take single pages of the rest
+    mha_need = int(nblk[0].sum())
+    mha_ids = supers[:mha_need] * 4
+    rest = np.concatenate([sp * 4 + np.arange(4) for sp in supers[mha_need:]])
+    rest = rest[rng.permutation(rest.size)]
+    gqa_ids = [rest[: int(nblk[1].sum())], rest[int(nblk[1].sum()) : int(nblk[1].sum()) + int(nblk[2].sum())]]
+    ids = [mha_ids] + gqa_ids
+    batches = []
+    for li, ((Hq, Hkv), pre, nb, blk) in enumerate(zip(COLOC_LAYOUTS, lens, nblk, ids)):
+        S = pre.size
+        max_blocks = int(nb.max())
+        table = np.full((S, max_blocks), -1, dtype=np.int32)
+        pos = 0
+        for s in range(S):
+            table[s, : nb[s]] = blk[pos : pos + nb[s]]
+            pos += int(nb[s])
+        q = bf16_normal(rng, (S, Hq, d))
+        k_new = bf16_normal(rng, (S, Hkv, d))
+        v_new = bf16_normal(rng, (S, Hkv, d))
+        batches.append(Batch(S=S, Hq=Hq, Hkv=Hkv, d=d, bs=bs, max_blocks=max_blocks, page_elems=page_elems,
+                             n_pages=n_pages, ctx_lens=(pre + 1).astype(np.int32), table=table, q=q,
+                             k_new=k_new, v_new=v_new, scale=1.0 / math.sqrt(d),
+                             meta={"seed": seed, "layout": li, "pre_lens": pre.copy()}))
+    pool = None
+    if fill_pool:
+        pool = np.empty(n_pages * page_elems, dtype=BF16)
+        bf16_normal_fill(pool, seed + 7919)
+    for b in batches:
+        b.pool = pool
+    return batches, n_pages, page_elems
+
+
+# ---------------------------------------------------------------------------
+# config 5: long-context heavy-tail stress
+# ---------------------------------------------------------------------------
+def config5_lengths(rng, n: int) -> np.ndarray:
+    """bounded Pareto(1.2) cached lengths on [256, 131072]"""
+    return bounded_pareto_lengths(rng, n, 1.2, 256, 131072)
+
+
+def config5_budgets(rng, n: int, lo: int = 1, hi: int = 64) -> np.ndarray:
+    """decode steps each sequence has left before it finishes (uniform)"""
+    return rng.integers(lo, hi + 1, size=n)
