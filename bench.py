@@ -6,8 +6,8 @@ lognormal context lengths with median 1024, sigma 1, clipped to 16384).
 A step is the whole hot path for one batch: the host sequence table advances
 every sequence by one token (growing reservations where needed) and syncs the
 lengths and changed table entries to the device, then the new K/V rows are
-appended and paged decode attention runs (attention kernel + split-K
-combine).  The headline
+appended and paged decode attention runs; by default the append is fused
+into the attention pass (one attention kernel + the split-K combine).  The headline
 value is algorithmic HBM GB/s of the step: K/V bytes read (each sequence's
 whole context) + q read + output written + appended K/V written, divided by
 the device time of the step.
@@ -182,6 +182,7 @@ def main():
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 CUDA cores, 2 tensor-core MMA")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -235,10 +236,13 @@ def main():
     def step(ev_pair=None):
         seqtab.advance()                         # host: every live sequence gains this step's token
         seqtab.sync(db.table, db.lens, stream)   # lengths (and any changed entries) to the device
-        db.append(stream)
         if ev_pair is not None:
             ev_pair[0].record(stream)
-        db.attend(stream=stream)
+        if args.separate_append:
+            db.append(stream)
+            db.attend(stream=stream)
+        else:
+            db.append_attend(stream)             # append fused into the attention pass
         if ev_pair is not None:
             ev_pair[1].record(stream)
         done[0] += 1
@@ -272,7 +276,7 @@ def main():
         ms = float(tt.item())
     err = pool.error(stream)
 
-    attn_bytes = [step_bytes(first + i)[0] for i in range(args.steps)]
+    attn_bytes = [step_bytes(first + i)[1] for i in range(args.steps)]  # the call also appends
     kv_total = sum(step_bytes(first + i)[1] for i in range(args.steps))
     gbs = kv_total / (ms * 1e-3) / 1e9 * world
     tokens_per_s = b.S * args.steps / (ms * 1e-3) * world
@@ -339,7 +343,7 @@ def main():
                      "peak_kind": peak_kind, "attn_ms": attn_avg_ms},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": (4 if args.separate_append else 3) * args.steps,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,

@@ -311,6 +311,21 @@ int paged_decode_attn(kv_pool *pool, int layout, const uint16_t *q, uint16_t *ou
                       size_t ws_bytes, void *stream);
 
 /*
+ * kv_append and paged_decode_attn in one pass (one launch fewer per step).
+ * The results are those of kv_append(k_new, v_new) followed by
+ * paged_decode_attn: the pool afterwards holds each sequence's new row at
+ * position n-1, and the attention uses it.  The warp that reads the tile
+ * holding position n-1 substitutes the new row in shared memory and then
+ * stores it to the pool, so no other reader sees the slot half-written.
+ * Sequences with n <= 0 or n beyond the table are not appended to.
+ * k_new, v_new: bf16 [S][Hkv][d] device arrays, 16-byte aligned.
+ */
+int paged_decode_attn_append(kv_pool *pool, int layout, const uint16_t *q, const uint16_t *k_new,
+                             const uint16_t *v_new, uint16_t *out, const int32_t *dev_table,
+                             const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale,
+                             int num_splits, void *workspace, size_t ws_bytes, void *stream);
+
+/*
  * paged_decode_attn for callers that cannot allocate device memory.  The
  * paper has no counterpart; this is a service of this library.  Callers that
  * cannot hand over a workspace include a server whose KV pool already holds

@@ -58,6 +58,9 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 struct AttnArgs {
     const uint16_t *q;
     uint16_t *out;
+    const uint16_t *k_new;   // fused append: this step's K/V rows [S][Hkv][d], or null
+    const uint16_t *v_new;
+    uint16_t *pool;          // pool base (rows of d bf16), for the fused append's writes
     const int32_t *table;
     const int32_t *ctx_lens;
     int32_t *err;
@@ -651,7 +654,17 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             const uint32_t par = consumed & 1u;
             const int nvalid = min(kTile, pc.n - (uu - pc.run_begin) * kTile);
             const bool more = uu + 1 < u1;
+            // fused append: the run's last tile holds position n-1, whose K/V
+            // row is this step's new token; this warp alone reads that tile
+            const bool app = a.k_new != nullptr && uu == pc.run_end - 1 && a.ctx_lens[pc.s] == pc.n;
+            const int arow = (pc.n - 1) % kTile;
             wait_phase(bk, par, a.err, dead);
+            if (app) {
+                if (lane < D / 8)
+                    *reinterpret_cast<uint4 *>(Ks + swz(arow, lane)) = *reinterpret_cast<const uint4 *>(
+                        a.k_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8);
+                __syncwarp();
+            }
             comp.qk(Ks, nvalid);
             // the K stage is refilled by TMA next: order the warp's generic
             // shared-memory reads before the async-proxy write
@@ -659,7 +672,25 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             __syncwarp();
             if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 0, k_addr, bk, policy);
             wait_phase(bv, par, a.err, dead);
+            if (app) {
+                if (lane < D / 8)
+                    *reinterpret_cast<uint4 *>(Vs + swz(arow, lane)) = *reinterpret_cast<const uint4 *>(
+                        a.v_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8);
+                __syncwarp();
+            }
             comp.pv(Vs);
+            if (app) {
+                // store the new row into the pool: this warp's own TMA reads of
+                // the tile have completed, and no other unit covers that row
+                const int32_t k = uu - cu0;
+                const int32_t y = k < a.rows_cap ? rows[k] : unit_row(a, T, uu);
+                if (y >= 0 && lane < D / 4) {
+                    const int which = lane / (D / 8), c = lane % (D / 8);
+                    const int64_t row = (int64_t)y + arow + (int64_t)which * Hkv * a.bs;
+                    const uint16_t *src = (which ? a.v_new : a.k_new) + ((int64_t)pc.s * Hkv + pc.g) * D + c * 8;
+                    *reinterpret_cast<uint4 *>(a.pool + row * D + c * 8) = *reinterpret_cast<const uint4 *>(src);
+                }
+            }
             fence_proxy_async_smem();
             __syncwarp();
             if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 1, v_addr, bv, policy);

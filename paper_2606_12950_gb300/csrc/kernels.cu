@@ -173,9 +173,13 @@ int kv_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int max_bloc
     return KV_OK;
 }
 
-int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, const int32_t *dev_table,
-                      const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale, int num_splits,
-                      void *workspace, size_t ws_bytes, void *stream)
+}  // extern "C"
+
+namespace {
+
+int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
+              uint16_t *out, const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq,
+              float scale, int num_splits, void *workspace, size_t ws_bytes, void *stream)
 {
     int G = 0;
     if (num_splits < 0 || !std::isfinite(scale)) return KV_ERR_INVALID_ARG;
@@ -183,12 +187,16 @@ int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, 
     if (rc) return rc;
     if (S == 0) return KV_OK;
     if (!q || !out || !dev_table || !dev_ctx_lens || !aligned16(q) || !aligned16(out)) return KV_ERR_INVALID_ARG;
+    if ((k_new || v_new) && (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))) return KV_ERR_INVALID_ARG;
     if (p->sm_count <= 0) return KV_ERR_CUDA;
     const kv_layout &L = p->desc.layouts[layout];
     const int variant = pick_variant(p, G);
     kvp::AttnArgs a{};
     a.q = q;
     a.out = out;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.pool = reinterpret_cast<uint16_t *>(p->desc.device_base);
     a.table = dev_table;
     a.ctx_lens = dev_ctx_lens;
     a.err = p->desc.device_error;
@@ -212,6 +220,28 @@ int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, 
     if (rc) return rc;
     return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                     true, &P);
+}
+
+}  // namespace
+
+extern "C" {
+
+int paged_decode_attn(kv_pool *p, int layout, const uint16_t *q, uint16_t *out, const int32_t *dev_table,
+                      const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale, int num_splits,
+                      void *workspace, size_t ws_bytes, void *stream)
+{
+    return attn_call(p, layout, q, nullptr, nullptr, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale,
+                     num_splits, workspace, ws_bytes, stream);
+}
+
+int paged_decode_attn_append(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new,
+                             const uint16_t *v_new, uint16_t *out, const int32_t *dev_table,
+                             const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale,
+                             int num_splits, void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!k_new || !v_new) return KV_ERR_INVALID_ARG;
+    return attn_call(p, layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale,
+                     num_splits, workspace, ws_bytes, stream);
 }
 
 }  // extern "C"

@@ -108,6 +108,7 @@ def lib() -> ctypes.CDLL:
             "kv_workspace_clear": [P, SZ, P],
             "paged_decode_attn": [P, I, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
+            "paged_decode_attn_append": [P, I, P, P, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "kv_set_attn_variant": [P, I],
             "kv_seqtab_create": [P, I, I, I, ctypes.POINTER(P)],
             "kv_seqtab_destroy": [P],
@@ -265,6 +266,17 @@ def paged_decode_attn(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_bl
            lib().paged_decode_attn(pool, layout, _addr(q), _addr(out), _addr(dev_table),
                                    _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq), float(scale),
                                    int(num_splits), _addr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def paged_decode_attn_append(pool, layout: int, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks: int,
+                             S: int, Hq: int, scale: float, num_splits: int, workspace, ws_bytes: int,
+                             stream=None) -> None:
+    """kv_append + paged_decode_attn fused into one pass."""
+    _check("paged_decode_attn_append",
+           lib().paged_decode_attn_append(pool, layout, _addr(q), _addr(k_new), _addr(v_new), _addr(out),
+                                          _addr(dev_table), _addr(dev_ctx_lens), int(max_blocks), int(S),
+                                          int(Hq), float(scale), int(num_splits), _addr(workspace),
+                                          int(ws_bytes), _stream(stream)))
 
 
 def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_blocks: int, S: int,

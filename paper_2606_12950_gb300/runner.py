@@ -109,6 +109,12 @@ class DeviceBatch:
                             self.max_blocks, self.S, self.Hq, self.b.scale, ns, self.ws,
                             self.ws.numel(), stream)
 
+    def append_attend(self, stream=None) -> None:
+        """The fused append + attention pass."""
+        K.paged_decode_attn_append(self.pool.handle, self.layout, self.q, self.k_new, self.v_new, self.out,
+                                   self.table, self.lens, self.max_blocks, self.S, self.Hq, self.b.scale,
+                                   self.num_splits, self.ws, self.ws.numel(), stream)
+
     def out_f64(self) -> np.ndarray:
         return self.out.float().cpu().numpy().astype(np.float64)
 

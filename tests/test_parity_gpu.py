@@ -26,15 +26,18 @@ def _cuda():
     from paper_2606_12950_gb300 import runner  # noqa: F401  (builds/loads libkvpool)
 
 
-def run(b, variant, num_splits=0, pool_u16=None):
+def run(b, variant, num_splits=0, pool_u16=None, fused=False):
     from paper_2606_12950_gb300.runner import DeviceBatch, DevicePool
 
     pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)])
     pool.upload(b.pool if pool_u16 is None else pool_u16)
     pool.set_variant(variant)
     db = DeviceBatch(pool, 0, b, num_splits)
-    db.append()
-    db.attend()
+    if fused:
+        db.append_attend()
+    else:
+        db.append()
+        db.attend()
     torch.cuda.synchronize()
     return pool, db
 
@@ -47,11 +50,12 @@ def check_attention(got, ref, what=""):
     return err
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("variant", VARIANTS)
 @pytest.mark.parametrize("num_splits", [0, 1, 3, 64])
-def test_config1_append_and_attention(variant, num_splits):
+def test_config1_append_and_attention(variant, num_splits, fused):
     b = W.config1_tiny()
-    pool, db = run(b, variant, num_splits)
+    pool, db = run(b, variant, num_splits, fused=fused)
     ref_pool = oracle.batch_append(b)
     assert np.array_equal(pool.download(), ref_pool), "pool after append differs"
     ref = oracle.batch_attention(b, pool=ref_pool)
@@ -70,14 +74,15 @@ SHAPES = [
 ]
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("variant", VARIANTS)
 @pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"G{s[0]}_Hkv{s[1]}_d{s[2]}_bs{s[3]}")
-def test_shapes_against_oracle(variant, shape):
+def test_shapes_against_oracle(variant, shape, fused):
     G, Hkv, d, bs, lens = shape
     if variant == 1 and G == 8:
         pytest.skip("the CUDA-core variant is built for G <= 5")
     b = W.make_batch(500 + G * 7 + d + bs, lens, Hq=G * Hkv, Hkv=Hkv, d=d, bs=bs, extra_blocks=9)
-    pool, db = run(b, variant)
+    pool, db = run(b, variant, fused=fused)
     ref_pool = oracle.batch_append(b)
     assert np.array_equal(pool.download(), ref_pool)
     ref = oracle.batch_attention(b, pool=ref_pool)
@@ -170,8 +175,9 @@ def test_device_bounds_check_sets_error_word(variant):
     assert pool.error() == 0  # read-and-clear
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("variant", VARIANTS)
-def test_decode_steps_track_the_oracle(variant):
+def test_decode_steps_track_the_oracle(variant, fused):
     """Several append+attend steps with growing lengths (including block
     boundaries), fresh q/k/v each step."""
     b = W.make_batch(95, [14, 15, 31, 47], Hq=8, Hkv=2, d=128, bs=16, table_tokens=np.array([64] * 4))
@@ -187,8 +193,11 @@ def test_decode_steps_track_the_oracle(variant):
         q, kn, vn = W.step_rows(95, step, b.S, b.Hq, b.Hkv, b.d)
         db.set_rows(q, kn, vn)
         db.upload_table(b.table, lens)
-        db.append()
-        db.attend()
+        if fused:
+            db.append_attend()
+        else:
+            db.append()
+            db.attend()
         torch.cuda.synchronize()
         host_pool = oracle.append(host_pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens)
         ref = oracle.paged_attention(host_pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, q, b.table, lens,
@@ -198,13 +207,14 @@ def test_decode_steps_track_the_oracle(variant):
     assert np.array_equal(pool.download(), host_pool)
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["separate", "fused"])
 @pytest.mark.parametrize("variant", VARIANTS)
-def test_llama8b_layer_full_size(variant):
+def test_llama8b_layer_full_size(variant, fused):
     """The Llama-3-8B-shaped layer (64 sequences, 32 q / 8 KV heads, d=128,
     bs=16, lognormal lengths) at full size in the benchmark's launch
     configuration, every sequence against the oracle."""
     b = W.config2_llama8b()
-    pool, db = run(b, variant)
+    pool, db = run(b, variant, fused=fused)
     ref_pool = oracle.batch_append(b)
     got_pool = pool.download()
     assert np.array_equal(got_pool, ref_pool)
