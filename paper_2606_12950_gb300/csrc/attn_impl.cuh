@@ -565,6 +565,10 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         fence_mbar_init();
     }
     if (tid == 32) prefetch_tensormap(&tmap);
+    // launched as a programmatic dependent: everything above touches only
+    // this CTA; wait here for the grid before (lengths, table, pool writes)
+    grid_launch_dependents();
+    grid_dependency_wait();
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {
@@ -748,6 +752,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
     __shared__ float s_L[kCombineThreads];
     const int r = blockIdx.x / CB, cb = blockIdx.x % CB;
     const int s = r / c.Hkv, g = r % c.Hkv;
+    grid_dependency_wait();  // the attention grid's partials and split index
     const int64_t W = c.ws_T[c.S], NP = c.ws_T[c.S + 1];
     if (W == 0) return;
     const int32_t nt = (c.ws_T[s + 1] - c.ws_T[s]) / c.Hkv;

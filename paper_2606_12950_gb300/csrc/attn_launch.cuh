@@ -34,11 +34,27 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     if (!launch) return KV_OK;
     a.rows_cap = kRowsCap;
     a.P = P;
-    fn<<<P, kThreads, smem, st>>>(*tmap, a);
-    if (cudaGetLastError() != cudaSuccess) return KV_ERR_CUDA;
+    // both kernels are programmatic dependents of what precedes them in the
+    // stream: they may be scheduled early and wait on the device
+    // (griddepcontrol.wait) for the previous grid to complete
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)P);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
     CombineArgs c{a.out, a.ws_T, a.ws_part, a.S, a.Hkv};
-    combine_kernel<D, G><<<a.S * a.Hkv * combine_ctas_per_run<D, G>(), kCombineThreads, 0, st>>>(c);
-    return cudaGetLastError() == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    cudaLaunchConfig_t ccfg = cfg;
+    ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv * combine_ctas_per_run<D, G>()));
+    ccfg.blockDim = dim3(kCombineThreads);
+    ccfg.dynamicSmemBytes = 0;
+    if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G>, c) != cudaSuccess) return KV_ERR_CUDA;
+    return KV_OK;
 }
 
 }  // namespace kvp

@@ -24,6 +24,9 @@ struct SyncParams {
 template <int WORDS>
 __global__ void seqtab_sync_kernel(const __grid_constant__ SyncParams<WORDS> p)
 {
+    // a following programmatic-dependent grid may launch now; it waits for
+    // this grid to complete before it reads the table or the lengths
+    asm volatile("griddepcontrol.launch_dependents;" :::);
     for (int i = threadIdx.x; i < p.n_lens; i += blockDim.x) p.dev_lens[p.lens_begin + i] = p.data[i];
     for (int j = threadIdx.x; j < p.n_patches; j += blockDim.x)
         p.dev_table[p.data[p.n_lens + 2 * j]] = p.data[p.n_lens + 2 * j + 1];
