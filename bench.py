@@ -104,13 +104,6 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def algorithmic_bytes(b):
-    kv = int(np.sum(b.ctx_lens.astype(np.int64))) * 2 * b.Hkv * b.d * 2
-    q_out = 2 * b.S * b.Hq * b.d * 2
-    app = 2 * b.S * b.Hkv * b.d * 2
-    return kv, q_out, app
-
-
 def oracle_baseline(b, budget_s: float):
     """Time the fp64 C oracle (single thread) on whole decode steps of the
     same workload (append + attention over every sequence) until budget_s
@@ -172,12 +165,168 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------------- workloads
+class Llama8B:
+    """Config 2: every sequence reserves its whole run up front (Eq. 2 with the
+    true total length); each step every sequence gains one token."""
+
+    name = WORKLOAD
+
+    def __init__(self, args, K, W, DevicePool, DeviceSteps):
+        total = 2 * (args.warmup + args.steps) + 8
+        b = W.config2_llama8b(steps=max(100, total))
+        self.b = b
+        self.pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)], shuffle_seed=b.meta["seed"])
+        self.pool.upload(b.pool)
+        if args.variant:
+            self.pool.set_variant(args.variant)
+        self.tab = K.SeqTab(self.pool.handle, 0, b.S, b.max_blocks)
+        self.pre = b.meta["pre_lens"].astype(np.int64)
+        for s in range(b.S):
+            self.tab.reserve(s, int(self.pre[s]) + total)
+            self.tab.set_len(s, int(self.pre[s]))
+        self.bufs = [DeviceSteps(self.pool, 0, b.S, b.S, b.Hq, b.Hkv, b.d, b.max_blocks, b.scale, b.q, b.k_new,
+                                 b.v_new, args.num_splits)]
+        self.S = b.S
+        self.config = {"S": b.S, "Hq": b.Hq, "Hkv": b.Hkv, "d": b.d, "bs": b.bs,
+                       "l2": "inputs larger than L2 (K+V ~ 326 MB per step; no flush needed)"}
+
+    def host_step(self):
+        self.tab.advance()
+        n = self.tab.lens().astype(np.int64)
+        kv = int(n.sum()) * 2 * self.b.Hkv * self.b.d * 2
+        other = 2 * self.b.S * self.b.Hq * self.b.d * 2 + 2 * self.b.S * self.b.Hkv * self.b.d * 2
+        return kv + other, kv + other  # (DRAM-algorithmic, logical) bytes
+
+    def tables(self):
+        return [(self.tab, self.bufs[0])]
+
+
+class Chains:
+    """Config 3: 256 Planner->Coder->Reviewer chains sharing a 2048-token
+    prefix; the prefix is counted once per step for the DRAM roofline."""
+
+    def __init__(self, args, K, W, DevicePool, DeviceSteps):
+        from paper_2606_12950_gb300.schedules import AgentChains
+
+        seed, n, d, Hq, Hkv, bs = 1003, 256, 128, 32, 8, 16
+        self.name = ("agent-chains: 256 Planner->Coder->Reviewer chains, 32 q / 8 kv, d=128, bs=16, shared "
+                     "2048-token prefix, stage outputs lognormal(300), reservations true x U[0.8,1.5]")
+        max_blocks = (W.PREFIX_TOKENS + 4 * 4096 * 2) // bs + 8
+        n_pages = 128 + n * 150 + 64
+        page_elems = 2 * Hkv * bs * d
+        host = np.empty(n_pages * page_elems, np.uint16)
+        W.bf16_normal_fill(host, seed + 7919)
+        self.pool = DevicePool(n_pages, page_elems * 2, bs, [(Hkv, d)], shuffle_seed=seed)
+        self.pool.upload(host)
+        del host
+        if args.variant:
+            self.pool.set_variant(args.variant)
+        self.ch = AgentChains(self.pool.handle, 0, n, max_blocks, bs, seed)
+        q, kn, vn = W.step_rows(seed, 0, n, Hq, Hkv, d)
+        self.bufs = [DeviceSteps(self.pool, 0, n + 1, n, Hq, Hkv, d, max_blocks, d ** -0.5, q, kn, vn,
+                                 args.num_splits)]
+        self.S, self.Hq, self.Hkv, self.d = n, Hq, Hkv, d
+        self.config = {"S": n, "Hq": Hq, "Hkv": Hkv, "d": d, "bs": bs,
+                       "l2": "private K+V larger than L2; the 8.4 MB shared prefix is meant to hit in L2"}
+
+    def host_step(self):
+        self.ch.step()
+        n = self.ch.ctx
+        per_tok = 2 * self.Hkv * self.d * 2
+        other = 2 * self.S * self.Hq * self.d * 2 + 2 * self.S * self.Hkv * self.d * 2
+        unique = (int((n - W_PREFIX).sum()) + W_PREFIX) * per_tok
+        logical = int(n.sum()) * per_tok
+        return unique + other, logical + other
+
+    def tables(self):
+        return [(self.ch.tab, self.bufs[0])]
+
+
+class Coloc:
+    """Config 4: three co-located layouts in one 90%-full pool; the same
+    decode step (append + attention per layout) is repeated."""
+
+    def __init__(self, args, K, W, DevicePool, DeviceSteps):
+        self.name = ("co-location: 512 seqs over MHA 32/32, GQA 32/8, GQA 40/8 (d=128, bs=16) in one pool "
+                     "filled to 90%, bounded Pareto(1.5) on [128, 32768]")
+        batches, n_pages, page_elems = W.config4_colocation()
+        self.pool = DevicePool(n_pages, page_elems * 2, 16, [(b.Hkv, b.d) for b in batches])
+        self.pool.upload(batches[0].pool)
+        if args.variant:
+            self.pool.set_variant(args.variant)
+        self.tabs, self.bufs = [], []
+        for li, b in enumerate(batches):
+            buf = DeviceSteps(self.pool, li, b.S, b.S, b.Hq, b.Hkv, b.d, b.max_blocks, b.scale, b.q, b.k_new,
+                              b.v_new, args.num_splits)
+            K.kv_block_table_upload(self.pool.handle, li, b.table, b.ctx_lens, buf.table, buf.lens)
+            self.bufs.append(buf)
+        self.batches = batches
+        self.S = sum(b.S for b in batches)
+        self.config = {"S": self.S, "layouts": [[b.Hq, b.Hkv, b.d] for b in batches], "bs": 16,
+                       "pool_gb": n_pages * page_elems * 2 / 1e9, "l2": "inputs larger than L2"}
+
+    def host_step(self):
+        tot = 0
+        for b in self.batches:
+            tot += int(b.ctx_lens.astype(np.int64).sum()) * 2 * b.Hkv * b.d * 2
+            tot += 2 * b.S * b.Hq * b.d * 2 + 2 * b.S * b.Hkv * b.d * 2
+        return tot, tot
+
+    def tables(self):
+        return [(None, buf) for buf in self.bufs]
+
+
+class LongCtx:
+    """Config 5: 1024 heavy-tailed sequences that finish and are replaced."""
+
+    def __init__(self, args, K, W, DevicePool, DeviceSteps):
+        from paper_2606_12950_gb300.schedules import LongContextStress
+
+        seed, S, d, Hq, Hkv, bs = 1005, 1024, 128, 32, 8, 32
+        self.name = ("long-context stress: 1024 seqs, 32 q / 8 kv, d=128, bs=32, bounded Pareto(1.2) on "
+                     "[256, 131072], sequences finish and are replaced")
+        max_blocks = (131072 + 64) // bs + 2
+        est = int(W.config5_lengths(np.random.default_rng(seed), S).sum())
+        n_pages = int(1.4 * est / bs) + 4096
+        page_elems = 2 * Hkv * bs * d
+        self.pool = DevicePool(n_pages, page_elems * 2, bs, [(Hkv, d)], shuffle_seed=seed)
+        # pool contents: seeded normal bf16 drawn on the device in one pass
+        # (timing only; the parity tests use host-drawn pools)
+        gen = __import__("torch").Generator(device="cuda").manual_seed(seed)
+        self.pool.buf.view(__import__("torch").bfloat16).normal_(generator=gen)
+        if args.variant:
+            self.pool.set_variant(args.variant)
+        self.lc = LongContextStress(self.pool.handle, 0, S, max_blocks, seed)
+        q, kn, vn = W.step_rows(seed, 0, S, Hq, Hkv, d)
+        self.bufs = [DeviceSteps(self.pool, 0, S, S, Hq, Hkv, d, max_blocks, d ** -0.5, q, kn, vn,
+                                 args.num_splits)]
+        self.S, self.Hq, self.Hkv, self.d = S, Hq, Hkv, d
+        self.config = {"S": S, "Hq": Hq, "Hkv": Hkv, "d": d, "bs": bs, "l2": "inputs larger than L2"}
+
+    def host_step(self):
+        self.lc.step()
+        n = self.lc.tab.lens().astype(np.int64)
+        live = int((n > 0).sum())
+        tot = int(n.sum()) * 2 * self.Hkv * self.d * 2 + 2 * live * self.Hq * self.d * 2 + \
+            2 * live * self.Hkv * self.d * 2
+        return tot, tot
+
+    def tables(self):
+        return [(self.lc.tab, self.bufs[0])]
+
+
+W_PREFIX = 2048
+WORKLOADS = {"llama8b": Llama8B, "chains": Chains, "coloc": Coloc, "longctx": LongCtx}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama8b", choices=sorted(WORKLOADS))
     ap.add_argument("--num-splits", type=int, default=0)
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 CUDA cores, 2 tensor-core MMA")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
@@ -206,46 +355,35 @@ def main():
 
     from paper_2606_12950_gb300 import kvpool as K
     from paper_2606_12950_gb300 import workloads as W
-    from paper_2606_12950_gb300.runner import DeviceBatch, DevicePool
+    from paper_2606_12950_gb300.runner import DevicePool, DeviceSteps
 
-    total_steps = 2 * (args.warmup + args.steps) + 8
-    b = W.config2_llama8b(steps=max(100, total_steps))
-    pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)], shuffle_seed=b.meta["seed"])
-    pool.upload(b.pool)
-    if args.variant:
-        pool.set_variant(args.variant)
-    db = DeviceBatch(pool, 0, b, args.num_splits)
+    wl = WORKLOADS[args.workload](args, K, W, DevicePool, DeviceSteps)
     stream = torch.cuda.current_stream()
-
-    # host sequence table: each sequence reserves its whole run up front
-    # (Eq. 2 with the true total length); blocks come from the shuffled pool
-    seqtab = K.SeqTab(pool.handle, 0, b.S, b.max_blocks)
-    pre = b.meta["pre_lens"].astype(np.int64)
-    for s in range(b.S):
-        seqtab.reserve(s, int(pre[s]) + total_steps)
-        seqtab.set_len(s, int(pre[s]))
-    done = [0]  # decode steps issued so far
-
-    def step_bytes(j):
-        """algorithmic bytes of decode step j: (attention call, whole step)"""
-        n = pre + 1 + j
-        kv = int(n.sum()) * 2 * b.Hkv * b.d * 2
-        qo = 2 * b.S * b.Hq * b.d * 2
-        return kv + qo, kv + qo + 2 * b.S * b.Hkv * b.d * 2
+    launches_per_step = 0
 
     def step(ev_pair=None):
-        seqtab.advance()                         # host: every live sequence gains this step's token
-        seqtab.sync(db.table, db.lens, stream)   # lengths (and any changed entries) to the device
+        """host bookkeeping, table sync, then append + attention per batch"""
+        nonlocal launches_per_step
+        nbytes = wl.host_step()
+        n = 0
+        for tab, buf in wl.tables():
+            if tab is not None:
+                tab.sync(buf.table, buf.lens, stream)
+                n += 1
         if ev_pair is not None:
             ev_pair[0].record(stream)
-        if args.separate_append:
-            db.append(stream)
-            db.attend(stream=stream)
-        else:
-            db.append_attend(stream)             # append fused into the attention pass
+        for _, buf in wl.tables():
+            if args.separate_append:
+                buf.append(stream)
+                buf.attend(stream)
+                n += 3
+            else:
+                buf.append_attend(stream)  # the append fused into the attention pass
+                n += 2
         if ev_pair is not None:
             ev_pair[1].record(stream)
-        done[0] += 1
+        launches_per_step = n
+        return nbytes
 
     for i in range(args.warmup):
         step()
@@ -261,10 +399,10 @@ def main():
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    first = done[0]
+    step_bytes = []
     t_start.record(stream)
     for i in range(args.steps):
-        step(evs[i])
+        step_bytes.append(step(evs[i]))
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -274,46 +412,53 @@ def main():
         tt = torch.tensor([ms], device="cuda")
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         ms = float(tt.item())
-    err = pool.error(stream)
+    err = wl.pool.error(stream)
 
-    attn_bytes = [step_bytes(first + i)[1] for i in range(args.steps)]  # the call also appends
-    kv_total = sum(step_bytes(first + i)[1] for i in range(args.steps))
-    gbs = kv_total / (ms * 1e-3) / 1e9 * world
-    tokens_per_s = b.S * args.steps / (ms * 1e-3) * world
+    dram_total = sum(x[0] for x in step_bytes)
+    logical_total = sum(x[1] for x in step_bytes)
+    gbs = dram_total / (ms * 1e-3) / 1e9 * world
+    tokens_per_s = wl.S * args.steps / (ms * 1e-3) * world
     attn_avg_ms = float(np.mean(attn_ms))
-    attn_gbs = float(np.mean(attn_bytes)) / (attn_avg_ms * 1e-3) / 1e9
+    attn_gbs = dram_total / args.steps / (attn_avg_ms * 1e-3) / 1e9
     peak, peak_kind = load_peaks()
 
-    # end to end: q / k / v from pinned host memory, output back to host
-    q_h = [torch.from_numpy(x.view(np.int16)).pin_memory() for x in W_step_rows(b, 0)]
-    out_h = torch.empty(db.out.shape, dtype=torch.bfloat16).pin_memory()
-    h2d = sum(int(t.numel()) * 2 for t in q_h) + b.S * 4
-    d2h = out_h.numel() * 2
+    # end to end: q / k / v from pinned host memory, output back to host, every step
+    bufs = [buf for _, buf in wl.tables()]
+    pinned = []
+    for buf in bufs:
+        pinned.append([torch.empty(t.shape, dtype=torch.bfloat16).pin_memory().copy_(t.cpu())
+                       for t in (buf.q, buf.k_new, buf.v_new)] +
+                      [torch.empty(buf.out.shape, dtype=torch.bfloat16).pin_memory()])
+    h2d = sum(int(p[i].numel()) * 2 for p in pinned for i in range(3)) + sum(b.rows * 4 for b in bufs)
+    d2h = sum(int(p[3].numel()) * 2 for p in pinned)
 
     def e2e_step():
-        db.q.view(torch.int16).copy_(q_h[0], non_blocking=True)
-        db.k_new.view(torch.int16).copy_(q_h[1], non_blocking=True)
-        db.v_new.view(torch.int16).copy_(q_h[2], non_blocking=True)
-        step()
-        out_h.copy_(db.out, non_blocking=True)
+        for buf, p in zip(bufs, pinned):
+            buf.q.copy_(p[0], non_blocking=True)
+            buf.k_new.copy_(p[1], non_blocking=True)
+            buf.v_new.copy_(p[2], non_blocking=True)
+        nb = step()
+        for buf, p in zip(bufs, pinned):
+            p[3].copy_(buf.out, non_blocking=True)
+        return nb
 
     for i in range(3):
         e2e_step()
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    first_e2e = done[0]
+    e2e_bytes = 0
     e0.record(stream)
     for i in range(args.steps):
-        e2e_step()
+        e2e_bytes += e2e_step()[0]
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_total = sum(step_bytes(first_e2e + i)[1] for i in range(args.steps))
     e2e_ms = e0.elapsed_time(e1)
-    e2e_gbs = e2e_total / (e2e_ms * 1e-3) / 1e9 * world
+    e2e_gbs = e2e_bytes / (e2e_ms * 1e-3) / 1e9 * world
 
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and not args.no_cpu_baseline and args.workload == "llama8b":
+        b = wl.b
         v, nst, el = oracle_baseline(b, args.cpu_budget)
         cpu = {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"{nst} whole decode steps (append + attention over all {b.S} sequences) of the same "
@@ -321,33 +466,34 @@ def main():
 
     traffic = None
     prof = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(prof):
+    if args.workload == "llama8b" and os.path.exists(prof):
         try:
             with open(prof) as f:
                 traffic = json.load(f).get("paged_attn_llama8b_bytes_per_launch")
         except Exception:
             traffic = None
 
+    config = {"workload": wl.name, **wl.config, "num_splits": args.num_splits, "variant": args.variant,
+              "append": "separate kernel" if args.separate_append else "fused into attention",
+              "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
     line = {
         "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "S": b.S, "Hq": b.Hq, "Hkv": b.Hkv, "d": b.d, "bs": b.bs,
-                   "context_tokens_first_step": int((pre + 1 + first).sum()),
-                   "kv_bytes_per_step": int(attn_bytes[0]), "l2": "inputs larger than L2 (no flush needed)",
-                   "num_splits": args.num_splits, "variant": args.variant,
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
         "decode_tokens_per_s": tokens_per_s,
         "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peak, "unit": "GB/s",
-                     "frac": attn_gbs / peak, "traffic": traffic, "kernel": "paged_attn_kernel",
+                     "frac": attn_gbs / peak, "traffic": traffic,
+                     "kernel": "paged_attn_kernel (+ combine_kernel, fused append)",
                      "peak_kind": peak_kind, "attn_ms": attn_avg_ms},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": (4 if args.separate_append else 3) * args.steps,
+        "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,
     }
+    if logical_total != dram_total:
+        line["logical_gbs"] = logical_total / (ms * 1e-3) / 1e9 * world
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:

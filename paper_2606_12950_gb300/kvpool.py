@@ -347,6 +347,13 @@ class SeqTab:
         lens = np.ctypeslib.as_array(ctypes.cast(l, ctypes.POINTER(ctypes.c_int32)), shape=(self.S,))
         return tab.reshape(self.S, self.max_blocks).copy(), lens.copy()
 
+    def lens(self) -> np.ndarray:
+        """Copy of the host lengths only."""
+        t = ctypes.c_void_p()
+        l = ctypes.c_void_p()
+        _check("kv_seqtab_host", lib().kv_seqtab_host(self.handle, ctypes.byref(t), ctypes.byref(l)))
+        return np.ctypeslib.as_array(ctypes.cast(l, ctypes.POINTER(ctypes.c_int32)), shape=(self.S,)).copy()
+
     def counters(self) -> dict:
         c = kv_seqtab_counters()
         _check("kv_seqtab_get_counters", lib().kv_seqtab_get_counters(self.handle, ctypes.byref(c)))

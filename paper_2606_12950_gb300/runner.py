@@ -120,3 +120,40 @@ class DeviceBatch:
 
     def out_bits(self) -> np.ndarray:
         return _host_u16(self.out)
+
+
+class DeviceSteps:
+    """Device buffers of a decode batch whose table and lengths come from a
+    host sequence table (rows >= S table rows; the first S rows decode)."""
+
+    def __init__(self, pool: DevicePool, layout: int, rows: int, S: int, Hq: int, Hkv: int, d: int,
+                 max_blocks: int, scale: float, q, k_new, v_new, num_splits: int = 0):
+        dev = pool.device
+        self.pool, self.layout = pool, layout
+        self.rows, self.S, self.Hq, self.Hkv, self.d = rows, S, Hq, Hkv, d
+        self.max_blocks, self.scale, self.num_splits = max_blocks, scale, num_splits
+        self.table = torch.full((rows, max_blocks), -1, dtype=torch.int32, device=dev)
+        self.lens = torch.zeros(rows, dtype=torch.int32, device=dev)
+        self.q = _dev_u16(q, dev)
+        self.k_new = _dev_u16(k_new, dev)
+        self.v_new = _dev_u16(v_new, dev)
+        self.out = torch.empty((S, Hq, d), dtype=torch.bfloat16, device=dev)
+        self.ws_bytes = K.kv_workspace_bytes(pool.handle, layout, S, Hq, max_blocks, num_splits)
+        self.ws = torch.empty(max(256, self.ws_bytes), dtype=torch.uint8, device=dev)
+
+    def sync(self, seqtab, stream=None) -> None:
+        seqtab.sync(self.table, self.lens, stream)
+
+    def append_attend(self, stream=None) -> None:
+        K.paged_decode_attn_append(self.pool.handle, self.layout, self.q, self.k_new, self.v_new, self.out,
+                                   self.table, self.lens, self.max_blocks, self.S, self.Hq, self.scale,
+                                   self.num_splits, self.ws, self.ws.numel(), stream)
+
+    def append(self, stream=None) -> None:
+        K.kv_append(self.pool.handle, self.layout, self.k_new, self.v_new, self.table, self.lens,
+                    self.max_blocks, self.S, stream)
+
+    def attend(self, stream=None) -> None:
+        K.paged_decode_attn(self.pool.handle, self.layout, self.q, self.out, self.table, self.lens,
+                            self.max_blocks, self.S, self.Hq, self.scale, self.num_splits, self.ws,
+                            self.ws.numel(), stream)

@@ -124,15 +124,14 @@ class LongContextStress:
         return True
 
     def step(self) -> None:
-        _, lens = self.tab.host()
-        for s in range(self.S):
-            if self.left[s] == 0:
-                if lens[s] > 0:
-                    self.tab.release(s)
-                    self.released += 1
-                self._admit(s)
-        _, lens = self.tab.host()
-        live = np.nonzero(lens > 0)[0].astype(np.int32)
+        lens = self.tab.lens()
+        for s in np.nonzero(self.left == 0)[0]:
+            s = int(s)
+            if lens[s] > 0:
+                self.tab.release(s)
+                self.released += 1
+            self._admit(s)
+        live = np.nonzero(self.tab.lens() > 0)[0].astype(np.int32)
         self.tab.advance(live)
         self.left[live] -= 1
 
