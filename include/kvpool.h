@@ -274,9 +274,9 @@ int kv_append(kv_pool *pool, int layout, const uint16_t *k_new, const uint16_t *
 
 /*
  * Bytes of device workspace paged_decode_attn needs for these sizes and this
- * num_splits: the batch's split index (S + 2 int32) followed by fp32 split
- * partials, one record of G*d + 2*G floats per (sequence, KV head, part)
- * pair a split run can produce.  Every call writes all it reads, so the
+ * num_splits: one (first part, part count) pair of int32 per (sequence, KV
+ * head) run, followed by fp32 split partials, one record of G*d + 2*G floats
+ * per (run, part) pair a split run can produce.  Every call writes all it reads, so the
  * workspace needs no initialisation and may be reused freely by calls that
  * are ordered on one stream.
  */

@@ -65,7 +65,7 @@ struct AttnArgs {
     const int32_t *ctx_lens;
     int32_t *err;
     float *ws_part;
-    int32_t *ws_T;           // T[0..S] and NP, for the combine kernel
+    int2 *ws_run;            // per run: (first part, parts) if split, else (part, 0)
     int64_t rows_per_page;   // page_bytes / (d * 2)
     int64_t pool_pages;
     int32_t pages_per_block;
@@ -581,6 +581,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             if (n == 0 && (s % a.P) == (int)blockIdx.x) {
                 // an empty context has no softmax: its output is defined as zero
                 for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
+                for (int g = 0; g < Hkv; ++g) a.ws_run[(int64_t)s * Hkv + g] = make_int2(0, 0);
             }
         }
         int32_t incl = local;
@@ -612,10 +613,6 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // exactly the parts part_of(first unit) .. part_of(last unit).
     const int64_t W = T[S];
     const int64_t NP = W < (int64_t)a.P * kWarps ? W : (int64_t)a.P * kWarps;
-    if (blockIdx.x == 0) {  // the combine kernel needs the same split
-        for (int i = tid; i <= S; i += kThreads) a.ws_T[i] = T[i];
-        if (tid == 0) a.ws_T[S + 1] = (int32_t)NP;
-    }
     const int64_t first_part = (int64_t)blockIdx.x * kWarps;
     if (first_part >= NP) return;
     const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
@@ -709,6 +706,8 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         uint16_t *orow = a.out + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D;
         float *slot = a.ws_part + ((int64_t)r + part) * MF;
         comp.store(orow, slot, split, lane);
+        if (part == p_first && lane == 0)  // each run has one first part: it tells the combine
+            a.ws_run[r] = make_int2(p_first, split ? p_last - p_first + 1 : 0);
         u = pc.pe;
     }
 }
@@ -723,7 +722,7 @@ constexpr int kCombineThreads = 256;
 
 struct CombineArgs {
     uint16_t *out;
-    const int32_t *ws_T;   // T[0..S], NP
+    const int2 *ws_run;    // per run: (first part, parts), parts = 0 when not split
     const float *ws_part;
     int32_t S;
     int32_t Hkv;
@@ -746,77 +745,58 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
     constexpr int CB = combine_ctas_per_run<D, G>();
     constexpr int NSPLIT = kCombineThreads / CW;   // thread groups splitting the partials
     static_assert(CW * CB == G * D / 4, "columns must tile the output");
-    __shared__ float s_max[kCombineThreads / 32][G];
-    __shared__ float s_M[G];
-    __shared__ float4 s_O[kCombineThreads];
+    __shared__ float s_M[kCombineThreads];
     __shared__ float s_L[kCombineThreads];
+    __shared__ float4 s_O[kCombineThreads];
     const int r = blockIdx.x / CB, cb = blockIdx.x % CB;
+    grid_dependency_wait();  // the attention grid's partials and run table
+    const int2 info = c.ws_run[r];
+    const int cnt = info.y;
+    if (cnt == 0) return;  // finished inside the attention kernel (or empty)
     const int s = r / c.Hkv, g = r % c.Hkv;
-    grid_dependency_wait();  // the attention grid's partials and split index
-    const int64_t W = c.ws_T[c.S], NP = c.ws_T[c.S + 1];
-    if (W == 0) return;
-    const int32_t nt = (c.ws_T[s + 1] - c.ws_T[s]) / c.Hkv;
-    if (nt == 0) return;
-    const int64_t run_begin = c.ws_T[s] + (int64_t)g * nt;
-    const int32_t p_first = cta_of(run_begin, W, NP);
-    const int32_t p_last = cta_of(run_begin + nt - 1, W, NP);
-    if (p_first == p_last) return;
-    const int cnt = p_last - p_first + 1;
-    const float *base = c.ws_part + ((int64_t)r + p_first) * MF;
+    const float *base = c.ws_part + ((int64_t)r + info.x) * MF;
     uint16_t *orow = c.out + ((int64_t)s * c.Hkv * G + (int64_t)g * G) * D;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-    // M_h = max over the partials, all (partial, head) pairs in parallel
-    float mx[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) mx[h] = -INFINITY;
-    for (int k = tid; k < cnt; k += kCombineThreads)
-#pragma unroll
-        for (int h = 0; h < G; ++h) mx[h] = fmaxf(mx[h], base[(int64_t)k * MF + G * D + h]);
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], off));
-        if (lane == 0) s_max[warp][h] = mx[h];
-    }
-    __syncthreads();
-    if (tid < G) {
-        float M = -INFINITY;
-        for (int w = 0; w < kCombineThreads / 32; ++w) M = fmaxf(M, s_max[w][tid]);
-        s_M[tid] = M;
-    }
-    __syncthreads();
-
-    // weighted sums: thread (group, column) takes partials group, group + NSPLIT, ...
+    const int tid = threadIdx.x;
     const int col = cb * CW + tid % CW;
     const int grp = tid / CW;
     const int h = (col * 4) / D;
-    const float M = s_M[h];
-    float L = 0.f;
+    // online merge of this group's partials (k = grp, grp + NSPLIT, ...):
+    // M running max, L and O relative to M
+    float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
+#pragma unroll 8
     for (int k = grp; k < cnt; k += NSPLIT) {
         const float *sl = base + (int64_t)k * MF;
-        const float sc = fast_exp2(sl[G * D + h] - M);
-        L += sc * sl[G * D + G + h];
-        const float4 o = *reinterpret_cast<const float4 *>(sl + col * 4);
-        O.x += sc * o.x;
-        O.y += sc * o.y;
-        O.z += sc * o.z;
-        O.w += sc * o.w;
+        const float mk = sl[G * D + h];
+        const float lk = sl[G * D + G + h];
+        const float4 ok = *reinterpret_cast<const float4 *>(sl + col * 4);
+        const float Mn = fmaxf(M, mk);
+        const float sa = fast_exp2(M - Mn), sb = fast_exp2(mk - Mn);
+        L = L * sa + lk * sb;
+        O.x = O.x * sa + ok.x * sb;
+        O.y = O.y * sa + ok.y * sb;
+        O.z = O.z * sa + ok.z * sb;
+        O.w = O.w * sa + ok.w * sb;
+        M = Mn;
     }
-    s_O[tid] = O;
+    s_M[tid] = M;
     s_L[tid] = L;
+    s_O[tid] = O;
     __syncthreads();
     if (grp == 0) {
-        // groups in order, so the sum order depends only on the run's shape
+        // merge the groups in order, so the result depends only on the run's shape
         for (int j = 1; j < NSPLIT; ++j) {
-            const float4 o = s_O[tid + j * CW];
-            O.x += o.x;
-            O.y += o.y;
-            O.z += o.z;
-            O.w += o.w;
-            L += s_L[tid + j * CW];
+            const float mj = s_M[tid + j * CW];
+            if (mj == -INFINITY) continue;  // group had no partials
+            const float Mn = fmaxf(M, mj);
+            const float sa = fast_exp2(M - Mn), sb = fast_exp2(mj - Mn);
+            const float4 oj = s_O[tid + j * CW];
+            L = L * sa + s_L[tid + j * CW] * sb;
+            O.x = O.x * sa + oj.x * sb;
+            O.y = O.y * sa + oj.y * sb;
+            O.z = O.z * sa + oj.z * sb;
+            O.w = O.w * sa + oj.w * sb;
+            M = Mn;
         }
         __nv_bfloat162 lo = __floats2bfloat162_rn(O.x / L, O.y / L);
         __nv_bfloat162 hi = __floats2bfloat162_rn(O.z / L, O.w / L);

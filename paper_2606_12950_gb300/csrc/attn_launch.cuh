@@ -48,7 +48,7 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
-    CombineArgs c{a.out, a.ws_T, a.ws_part, a.S, a.Hkv};
+    CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv};
     cudaLaunchConfig_t ccfg = cfg;
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv * combine_ctas_per_run<D, G>()));
     ccfg.blockDim = dim3(kCombineThreads);

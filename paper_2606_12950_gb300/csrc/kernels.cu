@@ -122,10 +122,11 @@ int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::Attn
     return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, launch, P_out);
 }
 
-// workspace: T[0..S] and NP (int32, padded to 256 bytes), then the partials
+// workspace: per-run (first part, parts) as int2 (padded to 256 bytes),
+// then the fp32 partials
 size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
 {
-    const size_t hdr = ((size_t)(S + 2) * 4 + 255) / 256 * 256;
+    const size_t hdr = ((size_t)S * Hkv * sizeof(int2) + 255) / 256 * 256;
     *part_off = hdr;
     return hdr + kvp::attn_partial_slots(S, Hkv, P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
@@ -214,7 +215,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     size_t part_off;
     const size_t need = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &part_off);
     if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
-    a.ws_T = reinterpret_cast<int32_t *>(workspace);
+    a.ws_run = reinterpret_cast<int2 *>(workspace);
     a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
