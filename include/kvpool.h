@@ -258,6 +258,113 @@ int kv_seqtab_host(const kv_seqtab *t, const int32_t **table, const int32_t **ct
 
 int kv_seqtab_get_counters(const kv_seqtab *t, kv_seqtab_counters *out);
 
+/* ---------------------------------------------------- memory accounting --- */
+
+/*
+ * Explicit memory accounting of a node runtime that colocates several models
+ * on one GPU (§III-C).  With M_total the GPU memory available to the runtime,
+ * M_kv the KV in use and, for every warm model k (Running or Sleeping), its
+ * persistent footprint M_ctx^k:
+ *     M_res = sum_k M_ctx^k + M_other,   safe iff M_kv + M_res <= M_total,
+ * and the KV admission headroom reported to the scheduler is
+ *     R_kv^head = M_total - M_res - M_kv.
+ * A model's persistent footprint is its kept runtime context (CUDA graphs,
+ * compiled kernels, buffers), plus its weights while those are on the GPU.
+ * Byte counts are the caller's; these calls touch no device memory.
+ */
+typedef enum kv_engine_state {
+    KV_ENGINE_IDLE = 0,          /* Running, no stage executing: weights + context on the GPU */
+    KV_ENGINE_SLEEPING = 1,      /* weights on the host, GPU context kept */
+    KV_ENGINE_SLEEP_PENDING = 2, /* a sleep transition has begun: weights + context still on the GPU */
+    KV_ENGINE_ACTIVE = 3,        /* Running with executing stages that hold KV */
+    KV_ENGINE_COLD = 4           /* CPU-, disk-resident or remote: nothing on the GPU, not warm */
+} kv_engine_state;
+
+typedef struct kv_engine {
+    int32_t state;             /* kv_engine_state */
+    int32_t reserved;          /* 0 */
+    uint64_t ctx_bytes;        /* kept runtime context (M_ctx without weights) */
+    uint64_t weight_bytes;     /* weights; on the GPU in IDLE, SLEEP_PENDING and ACTIVE */
+    uint64_t kv_bytes;         /* KV mapped for the engine's executing stages (ACTIVE only) */
+    uint64_t virtual_kv_bytes; /* the engine's virtual KV address space (may exceed physical) */
+    double weight_reload_s;    /* time to bring the weights back (profiled bandwidth) */
+    double ctx_rebuild_s;      /* time to rebuild the runtime context */
+    double kv_swap_in_s;       /* time to swap the engine's KV back in */
+    double kv_regen_s;         /* time to regenerate the engine's KV (profiled compute) */
+} kv_engine;
+
+typedef struct kv_account {
+    uint64_t m_res;            /* sum of warm footprints + M_other */
+    uint64_t m_kv;             /* kv_bytes of ACTIVE engines + extra_kv_bytes */
+    uint64_t m_kv_virtual;     /* virtual_kv_bytes of warm engines */
+    int64_t headroom;          /* R_kv^head = M_total - M_res - M_kv (negative when unsafe) */
+    int32_t safe;              /* M_kv + M_res <= M_total */
+    int32_t reserved;
+    double overcommit;         /* m_kv_virtual / M_total (0 when M_total is 0) */
+} kv_account;
+
+/*
+ * Account n engines.  extra_kv_bytes adds KV in use that no listed engine
+ * owns.  KV_ERR_INVALID_ARG for a null pointer, n < 0 or a bad state.
+ */
+int kv_memory_account(const kv_engine *engines, int n, uint64_t m_total, uint64_t m_other,
+                      uint64_t extra_kv_bytes, kv_account *out);
+
+typedef enum kv_degrade_action {
+    KV_ACT_SLEEP = 1,      /* level 1: an idle Running model goes to sleep; frees its weights */
+    KV_ACT_EVICT = 2,      /* level 2: a Sleeping model is evicted; frees its context */
+    KV_ACT_STOP = 3,       /* level 3: a pending sleep transition is stopped by shutting the
+                              engine down; frees weights + context */
+    KV_ACT_PREEMPT = 4,    /* level 4: an Active model's KV is swapped out to the host */
+    KV_ACT_ABORT = 5       /* level 5: an Active model's executions are aborted; frees their KV */
+} kv_degrade_action;
+
+typedef struct kv_plan_step {
+    int32_t engine;        /* index into the engines array */
+    int32_t action;        /* kv_degrade_action */
+    uint64_t freed_bytes;  /* estimated memory the action frees */
+    double cost_s;         /* c(e, a): restoration latency of the action */
+} kv_plan_step;
+
+/*
+ * Minimum-impact memory coordination (Alg. 2) and its disruption cost
+ * (Eq. 3).  Warm engines are visited level by level (IDLE, SLEEPING,
+ * SLEEP_PENDING, ACTIVE; within a level in array order, so pass them
+ * least-recently-used first) and each receives the least disruptive action
+ * its state allows, until the freed memory reaches `required` bytes:
+ *   IDLE -> SLEEP (frees weights, c = weight_reload_s);
+ *   SLEEPING -> EVICT (frees context, c = ctx_rebuild_s);
+ *   SLEEP_PENDING -> STOP (frees weights + context, c = weight_reload_s + ctx_rebuild_s);
+ *   ACTIVE -> PREEMPT while its KV fits the host swap space the plan has
+ *     left (c = kv_swap_in_s), else ABORT (c = kv_regen_s); both free the
+ *     KV and raise the interrupt flag.
+ * Engines whose action would free nothing, and COLD engines, are passed over.
+ *   C_deg = sum over the plan of c(e, a) + [interrupt] * c_int.
+ * Up to max_steps steps are written (n_steps counts all of them).  Returns
+ * KV_OK when the plan frees at least `required`, KV_ERR_OUT_OF_BLOCKS
+ * (infeasible: every engine was used and still less was freed; the steps
+ * are still written), KV_ERR_INVALID_ARG for bad arguments.  required = 0
+ * gives an empty plan with C_deg = 0.
+ */
+int kv_degradation_plan(const kv_engine *engines, int n, uint64_t required, uint64_t host_swap_bytes,
+                        double c_int, kv_plan_step *steps, int max_steps, int *n_steps, int *interrupt,
+                        double *c_deg, uint64_t *freed);
+
+/*
+ * Admission check of a stage that needs `demand` more bytes of KV (§III-C).
+ * If demand <= R_kv^head the stage fits: KV_OK with *n_steps = 0 and
+ * C_deg = 0.  Otherwise a degradation plan for R = demand - R_kv^head is
+ * derived as kv_degradation_plan does: KV_OK with *n_steps > 0 when the plan
+ * makes room (the caller executes it before admitting), KV_ERR_OUT_OF_BLOCKS
+ * when it cannot (the stage is rejected; the plan and C_deg still describe
+ * everything the node could free).  *headroom receives R_kv^head before any
+ * degradation.
+ */
+int kv_admission_check(const kv_engine *engines, int n, uint64_t m_total, uint64_t m_other,
+                       uint64_t extra_kv_bytes, uint64_t demand, uint64_t host_swap_bytes, double c_int,
+                       kv_plan_step *steps, int max_steps, int *n_steps, int *interrupt, double *c_deg,
+                       int64_t *headroom);
+
 /* -------------------------------------------------------------- kernels --- */
 
 /*

@@ -78,6 +78,45 @@ class kv_stats(ctypes.Structure):
     ]
 
 
+class kv_engine(ctypes.Structure):
+    _fields_ = [
+        ("state", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+        ("ctx_bytes", ctypes.c_uint64),
+        ("weight_bytes", ctypes.c_uint64),
+        ("kv_bytes", ctypes.c_uint64),
+        ("virtual_kv_bytes", ctypes.c_uint64),
+        ("weight_reload_s", ctypes.c_double),
+        ("ctx_rebuild_s", ctypes.c_double),
+        ("kv_swap_in_s", ctypes.c_double),
+        ("kv_regen_s", ctypes.c_double),
+    ]
+
+
+class kv_account(ctypes.Structure):
+    _fields_ = [
+        ("m_res", ctypes.c_uint64),
+        ("m_kv", ctypes.c_uint64),
+        ("m_kv_virtual", ctypes.c_uint64),
+        ("headroom", ctypes.c_int64),
+        ("safe", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+        ("overcommit", ctypes.c_double),
+    ]
+
+
+class kv_plan_step(ctypes.Structure):
+    _fields_ = [
+        ("engine", ctypes.c_int32),
+        ("action", ctypes.c_int32),
+        ("freed_bytes", ctypes.c_uint64),
+        ("cost_s", ctypes.c_double),
+    ]
+
+
+KV_ENGINE_IDLE, KV_ENGINE_SLEEPING, KV_ENGINE_SLEEP_PENDING, KV_ENGINE_ACTIVE, KV_ENGINE_COLD = 0, 1, 2, 3, 4
+KV_ACT_SLEEP, KV_ACT_EVICT, KV_ACT_STOP, KV_ACT_PREEMPT, KV_ACT_ABORT = 1, 2, 3, 4, 5
+
 _lib = None
 
 
@@ -121,6 +160,12 @@ def lib() -> ctypes.CDLL:
             "kv_seqtab_sync": [P, P, P, P],
             "kv_seqtab_host": [P, ctypes.POINTER(P), ctypes.POINTER(P)],
             "kv_seqtab_get_counters": [P, ctypes.POINTER(kv_seqtab_counters)],
+            "kv_memory_account": [P, I, U64, U64, U64, ctypes.POINTER(kv_account)],
+            "kv_degradation_plan": [P, I, U64, U64, ctypes.c_double, P, I, ctypes.POINTER(I),
+                                    ctypes.POINTER(I), ctypes.POINTER(ctypes.c_double),
+                                    ctypes.POINTER(U64)],
+            "kv_admission_check": [P, I, U64, U64, U64, U64, U64, ctypes.c_double, P, I, ctypes.POINTER(I),
+                                   ctypes.POINTER(I), ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I64)],
         }
         for name, args in sigs.items():
             f = getattr(L, name)
@@ -364,3 +409,61 @@ class SeqTab:
             self.close()
         except Exception:
             pass
+
+
+def _engines(engines):
+    """A sequence of kv_engine or of dicts with kv_engine's field names."""
+    arr = (kv_engine * max(1, len(engines)))()
+    for i, e in enumerate(engines):
+        if isinstance(e, kv_engine):
+            arr[i] = e
+        else:
+            for k, v in e.items():
+                setattr(arr[i], k, v)
+    return arr
+
+
+def _steps(arr, n):
+    return [{"engine": arr[i].engine, "action": arr[i].action, "freed_bytes": arr[i].freed_bytes,
+             "cost_s": arr[i].cost_s} for i in range(n)]
+
+
+def kv_memory_account(engines, m_total: int, m_other: int, extra_kv_bytes: int = 0) -> dict:
+    arr = _engines(engines)
+    out = kv_account()
+    _check("kv_memory_account", lib().kv_memory_account(ctypes.addressof(arr), len(engines), m_total, m_other,
+                                                        extra_kv_bytes, ctypes.byref(out)))
+    return {"m_res": out.m_res, "m_kv": out.m_kv, "m_kv_virtual": out.m_kv_virtual, "headroom": out.headroom,
+            "safe": bool(out.safe), "overcommit": out.overcommit}
+
+
+def kv_degradation_plan(engines, required: int, host_swap_bytes: int = 0, c_int: float = 0.0) -> dict:
+    """Alg. 2 + Eq. 3.  Returns {ok, steps, interrupt, c_deg, freed}; ok is False
+    when the plan cannot free `required` (KV_ERR_OUT_OF_BLOCKS)."""
+    arr = _engines(engines)
+    cap = max(1, len(engines))
+    steps = (kv_plan_step * cap)()
+    n, intr, c, fr = ctypes.c_int(), ctypes.c_int(), ctypes.c_double(), ctypes.c_uint64()
+    rc = lib().kv_degradation_plan(ctypes.addressof(arr), len(engines), required, host_swap_bytes, c_int,
+                                   ctypes.addressof(steps), cap, ctypes.byref(n), ctypes.byref(intr),
+                                   ctypes.byref(c), ctypes.byref(fr))
+    if rc not in (KV_OK, KV_ERR_OUT_OF_BLOCKS):
+        raise KVError("kv_degradation_plan", rc)
+    return {"ok": rc == KV_OK, "steps": _steps(steps, n.value), "interrupt": bool(intr.value), "c_deg": c.value,
+            "freed": fr.value}
+
+
+def kv_admission_check(engines, m_total: int, m_other: int, extra_kv_bytes: int, demand: int,
+                       host_swap_bytes: int = 0, c_int: float = 0.0) -> dict:
+    """§III-C admission.  Returns {ok, steps, interrupt, c_deg, headroom}."""
+    arr = _engines(engines)
+    cap = max(1, len(engines))
+    steps = (kv_plan_step * cap)()
+    n, intr, c, h = ctypes.c_int(), ctypes.c_int(), ctypes.c_double(), ctypes.c_int64()
+    rc = lib().kv_admission_check(ctypes.addressof(arr), len(engines), m_total, m_other, extra_kv_bytes, demand,
+                                  host_swap_bytes, c_int, ctypes.addressof(steps), cap, ctypes.byref(n),
+                                  ctypes.byref(intr), ctypes.byref(c), ctypes.byref(h))
+    if rc not in (KV_OK, KV_ERR_OUT_OF_BLOCKS):
+        raise KVError("kv_admission_check", rc)
+    return {"ok": rc == KV_OK, "steps": _steps(steps, n.value), "interrupt": bool(intr.value), "c_deg": c.value,
+            "headroom": h.value}
