@@ -242,6 +242,9 @@ class Chains:
     def tables(self):
         return [(self.ch.tab, self.bufs[0])]
 
+    def prefix_plan(self):
+        return self.ch.prefix_plan()
+
 
 class Coloc:
     """Config 4: three co-located layouts in one 90%-full pool; the same
@@ -332,6 +335,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
+    ap.add_argument("--no-cascade", action="store_true",
+                    help="agent chains: stream the shared prefix per chain instead of once per KV head")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -360,6 +365,11 @@ def main():
     wl = WORKLOADS[args.workload](args, K, W, DevicePool, DeviceSteps)
     stream = torch.cuda.current_stream()
     launches_per_step = 0
+    cascade = None
+    if hasattr(wl, "prefix_plan") and not args.no_cascade and not args.separate_append:
+        cascade = wl.prefix_plan()
+        for _, buf in wl.tables():
+            buf.use_cascade()
 
     def step(ev_pair=None):
         """host bookkeeping, table sync, then append + attention per batch"""
@@ -373,7 +383,10 @@ def main():
         if ev_pair is not None:
             ev_pair[0].record(stream)
         for _, buf in wl.tables():
-            if args.separate_append:
+            if cascade is not None:
+                buf.cascade(cascade, stream=stream)  # prefix kernel + attention (fused append) + combine
+                n += 3
+            elif args.separate_append:
                 buf.append(stream)
                 buf.attend(stream)
                 n += 3
@@ -475,6 +488,8 @@ def main():
 
     config = {"workload": wl.name, **wl.config, "num_splits": args.num_splits, "variant": args.variant,
               "append": "separate kernel" if args.separate_append else "fused into attention",
+              "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
+                                else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,
               "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
     line = {
         "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world, "steps": args.steps,

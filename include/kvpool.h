@@ -433,6 +433,48 @@ int paged_decode_attn_append(kv_pool *pool, int layout, const uint16_t *q, const
                              int num_splits, void *workspace, size_t ws_bytes, void *stream);
 
 /*
+ * Shared-prefix ("cascade") decode attention.  Sequences that hold the same
+ * physical blocks at the start of their block tables -- a system prompt
+ * shared by reference by every stage of an agent workflow (§III-B, §III-C)
+ * -- have identical K/V for those tokens.  For every group of such
+ * sequences, the prefix's attention is computed once per KV head for all
+ * members together as a dense tensor-core contraction, each member's own
+ * suffix is streamed as in paged_decode_attn (with the fused append when
+ * k_new / v_new are given, as paged_decode_attn_append), and the two are
+ * merged exactly (the softmax factorises over a partition of the keys).
+ * The result equals paged_decode_attn's on the same inputs, up to rounding.
+ *
+ * groups[i] = {count, tokens}: group i's members are the next `count`
+ * entries of members[] (host arrays, groups in order); `tokens` is the
+ * shared prefix length, a multiple of 64 and of the block size, at most
+ * max_blocks * bs.  The prefix blocks are read from the first member's
+ * table row; the caller guarantees every member's first tokens/bs entries
+ * are the same blocks and, when appending, that every member's length
+ * (post-append) exceeds tokens (so the new token never lands in a shared
+ * block).  A member whose length equals tokens (no append) attends over the
+ * prefix alone.  A sequence is in at most one group; sequences in no group
+ * are computed as by paged_decode_attn.  n_groups = 0 is paged_decode_attn
+ * (or _append).  The plan travels as kernel parameters:
+ *     3 * n_groups + 2 + (members) + S <= 4080 words.
+ * Workspace: kv_cascade_workspace_bytes() (256-byte aligned).
+ * Errors: KV_ERR_INVALID_ARG (bad plan, duplicate member, words over the
+ * limit), KV_ERR_WORKSPACE, KV_ERR_UNSUPPORTED, KV_ERR_CUDA; on the device a
+ * member shorter than its prefix sets KV_ERR_DEVICE_BOUNDS in the error word.
+ */
+typedef struct kv_prefix_group {
+    int32_t count;   /* members in the group */
+    int32_t tokens;  /* shared prefix tokens */
+} kv_prefix_group;
+
+int kv_cascade_workspace_bytes(const kv_pool *pool, int layout, int S, int Hq, int max_blocks, size_t *out_bytes);
+
+int paged_decode_attn_cascade(kv_pool *pool, int layout, const uint16_t *q, const uint16_t *k_new,
+                              const uint16_t *v_new, uint16_t *out, const int32_t *dev_table,
+                              const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale,
+                              const kv_prefix_group *groups, int n_groups, const int32_t *members, void *workspace,
+                              size_t ws_bytes, void *stream);
+
+/*
  * paged_decode_attn for callers that cannot allocate device memory.  The
  * paper has no counterpart; this is a service of this library.  Callers that
  * cannot hand over a workspace include a server whose KV pool already holds

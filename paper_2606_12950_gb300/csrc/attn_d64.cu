@@ -23,3 +23,17 @@ int kvp_attn_d64(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArg
     }
 #undef KVP_CASE
 }
+
+int kvp_cascade_d64(int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sm_count,
+                    cudaStream_t st, bool launch, int *P_out)
+{
+    using namespace kvp;
+    switch (G) {
+    case 1: return cascade_run<64, 1>(tmap, c, grid, sm_count, st, launch, P_out);
+    case 2: return cascade_run<64, 2>(tmap, c, grid, sm_count, st, launch, P_out);
+    case 4: return cascade_run<64, 4>(tmap, c, grid, sm_count, st, launch, P_out);
+    case 5: return cascade_run<64, 5>(tmap, c, grid, sm_count, st, launch, P_out);
+    case 8: return cascade_run<64, 8>(tmap, c, grid, sm_count, st, launch, P_out);
+    default: return KV_ERR_UNSUPPORTED;
+    }
+}

@@ -76,6 +76,12 @@ struct AttnArgs {
     int32_t rows_cap;        // units whose pool rows are resolved up front
     int32_t P;               // CTAs (work partitions)
     float qk_scale;          // scale * log2(e)
+    // shared-prefix (cascade) mode: tokens of each sequence's prefix handled
+    // by the prefix kernel ([S], multiples of 16; null = none), its records
+    // and key-split count (read by the combine)
+    const int32_t *skip;
+    const float *ws_pre;
+    int32_t KS;
 };
 
 __device__ __forceinline__ void report(int32_t *err, int code) { atomicCAS(err, 0, code); }
@@ -455,6 +461,7 @@ struct Piece {
     int32_t run_begin;     // unit id of tile 0 of this (s, g) run
     int32_t run_end;
     int32_t s, g, n;       // sequence, KV head, context length
+    int32_t skip;          // leading tokens handled by the prefix kernel
 };
 
 __device__ __forceinline__ int32_t clamp_len(const AttnArgs &a, int s, bool report_errors)
@@ -466,6 +473,30 @@ __device__ __forceinline__ int32_t clamp_len(const AttnArgs &a, int s, bool repo
         n = n < 0 ? 0 : cap;
     }
     return n;
+}
+
+// leading tokens of sequence s (context n) left to the prefix kernel: 0
+// outside cascade mode; a value that is not a multiple of 16 in [0, n] is
+// reported and clamped
+__device__ __forceinline__ int32_t seq_skip(const AttnArgs &a, int s, int32_t n, bool report_errors)
+{
+    if (!a.skip) return 0;
+    int32_t k = a.skip[s];
+    if (k < 0 || k > n || (k % kTile)) {
+        if (report_errors) report(a.err, KV_ERR_DEVICE_BOUNDS);
+        k = k < 0 ? 0 : (k > n ? n : k);
+        k -= k % kTile;
+    }
+    return k;
+}
+
+// units of sequence s: 16-token tiles of its (suffix) context, per KV head
+__device__ __forceinline__ int32_t seq_units(const AttnArgs &a, int s, bool report_errors, int32_t *ne_out)
+{
+    const int32_t n = clamp_len(a, s, report_errors);
+    const int32_t ne = n - seq_skip(a, s, n, report_errors);
+    if (ne_out) *ne_out = ne;
+    return ((ne + kTile - 1) / kTile) * a.Hkv;
 }
 
 // largest s with T[s] <= u; T[s] = first unit of sequence s, T[S] = total,
@@ -488,6 +519,7 @@ __device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T
     p.s = s;
     p.g = g;
     p.n = clamp_len(a, s, false);
+    p.skip = seq_skip(a, s, p.n, false);
     p.run_begin = T[s] + g * nt;
     p.run_end = p.run_begin + nt;
     p.pb = u;
@@ -502,7 +534,7 @@ __device__ __forceinline__ int32_t unit_row(const AttnArgs &a, const int32_t *T,
     const int32_t nt = (T[s + 1] - T[s]) / a.Hkv;
     const int32_t within = u - T[s];
     const int32_t g = within / nt;
-    const int32_t tok0 = (within - g * nt) * kTile;
+    const int32_t tok0 = seq_skip(a, s, clamp_len(a, s, false), false) + (within - g * nt) * kTile;
     const int32_t phys = a.table[(int64_t)s * a.max_blocks + tok0 / a.bs];
     if (phys < 0 || (int64_t)phys + a.pages_per_block > a.pool_pages) return -1;
     return (int32_t)((int64_t)phys * a.rows_per_page + (tok0 % a.bs) + (int64_t)g * a.bs);
@@ -576,11 +608,17 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         const int lo = min(S, tid * per), hi = min(S, lo + per);
         int32_t local = 0;
         for (int s = lo; s < hi; ++s) {
-            const int32_t n = clamp_len(a, s, true);
-            local += ((n + kTile - 1) / kTile) * Hkv;
-            if (n == 0 && (s % a.P) == (int)blockIdx.x) {
-                // an empty context has no softmax: its output is defined as zero
-                for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
+            int32_t ne;
+            local += seq_units(a, s, true, &ne);
+            // the fused append needs the new token outside a shared prefix
+            if (ne == 0 && a.skip && a.k_new && clamp_len(a, s, false) > 0 && (s % a.P) == (int)blockIdx.x)
+                report(a.err, KV_ERR_DEVICE_BOUNDS);
+            if (ne == 0 && (s % a.P) == (int)blockIdx.x) {
+                // an empty context has no softmax: its output is defined as
+                // zero; a sequence whose whole context is a shared prefix
+                // gets its output from the prefix records alone
+                if (clamp_len(a, s, false) == 0)
+                    for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
                 for (int g = 0; g < Hkv; ++g) a.ws_run[(int64_t)s * Hkv + g] = make_int2(0, 0);
             }
         }
@@ -597,7 +635,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         int32_t run = base + incl - local;
         for (int s = lo; s < hi; ++s) {
             T[s] = run;
-            run += ((clamp_len(a, s, false) + kTile - 1) / kTile) * Hkv;
+            run += seq_units(a, s, false, nullptr);
         }
         if (tid == 0) {
             int32_t tot = 0;
@@ -653,7 +691,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         comp.begin(a.q + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D, a.qk_scale, lane);
         for (int32_t uu = pc.pb; uu < pc.pe; ++uu) {
             const uint32_t par = consumed & 1u;
-            const int nvalid = min(kTile, pc.n - (uu - pc.run_begin) * kTile);
+            const int nvalid = min(kTile, pc.n - pc.skip - (uu - pc.run_begin) * kTile);
             const bool more = uu + 1 < u1;
             // fused append: the run's last tile holds position n-1, whose K/V
             // row is this step's new token; this warp alone reads that tile
@@ -702,7 +740,8 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         const int32_t r = pc.s * Hkv + pc.g;
         const int32_t p_first = cta_of(pc.run_begin, W, NP);
         const int32_t p_last = cta_of(pc.run_end - 1, W, NP);
-        const bool split = p_first != p_last;
+        // a run whose prefix lives in prefix records always leaves a partial
+        const bool split = p_first != p_last || pc.skip > 0;
         uint16_t *orow = a.out + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D;
         float *slot = a.ws_part + ((int64_t)r + part) * MF;
         comp.store(orow, slot, split, lane);
@@ -726,6 +765,9 @@ struct CombineArgs {
     const float *ws_part;
     int32_t S;
     int32_t Hkv;
+    const int32_t *skip;   // cascade mode: sequences with skip > 0 also merge
+    const float *ws_pre;   // KS prefix records [k][S][Hkv], ahead of their parts
+    int32_t KS;
 };
 
 // columns (float4 of o) per combine CTA, and CTAs per run
@@ -751,9 +793,10 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
     const int r = blockIdx.x / CB, cb = blockIdx.x % CB;
     grid_dependency_wait();  // the attention grid's partials and run table
     const int2 info = c.ws_run[r];
-    const int cnt = info.y;
-    if (cnt == 0) return;  // finished inside the attention kernel (or empty)
     const int s = r / c.Hkv, g = r % c.Hkv;
+    const int npre = (c.skip != nullptr && c.skip[s] > 0) ? c.KS : 0;
+    const int cnt = info.y + npre;
+    if (cnt == 0) return;  // finished inside the attention kernel (or empty)
     const float *base = c.ws_part + ((int64_t)r + info.x) * MF;
     uint16_t *orow = c.out + ((int64_t)s * c.Hkv * G + (int64_t)g * G) * D;
     const int tid = threadIdx.x;
@@ -766,7 +809,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
     for (int k = grp; k < cnt; k += NSPLIT) {
-        const float *sl = base + (int64_t)k * MF;
+        const float *sl = k < npre ? c.ws_pre + (((int64_t)k * c.S + s) * c.Hkv + g) * MF
+                                   : base + (int64_t)(k - npre) * MF;
         const float mk = sl[G * D + h];
         const float lk = sl[G * D + G + h];
         const float4 ok = *reinterpret_cast<const float4 *>(sl + col * 4);

@@ -6,7 +6,7 @@
 #include <algorithm>
 #include <atomic>
 
-#include "attn_impl.cuh"
+#include "cascade_impl.cuh"
 
 namespace kvp {
 
@@ -48,13 +48,47 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
-    CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv};
+    CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv, a.skip, a.ws_pre, a.KS};
     cudaLaunchConfig_t ccfg = cfg;
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv * combine_ctas_per_run<D, G>()));
     ccfg.blockDim = dim3(kCombineThreads);
     ccfg.dynamicSmemBytes = 0;
     if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G>, c) != cudaSuccess) return KV_ERR_CUDA;
     return KV_OK;
+}
+
+// Shared-prefix kernel: with launch = false only reports the CTAs that fit
+// on the GPU at once (occupancy x SMs) in *P_out.
+template <int D, int G>
+int cascade_run(const CUtensorMap *tmap, const CascadeArgs *c, int grid, int sm_count, cudaStream_t st, bool launch,
+                int *P_out)
+{
+    auto fn = cascade_prefix_kernel<D, G>;
+    const size_t smem = cascade_smem_bytes<D>();
+    static std::atomic<bool> attr_set{false};
+    if (!attr_set.load()) {
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+            return KV_ERR_CUDA;
+        attr_set.store(true);
+    }
+    if (!launch) {
+        int occ = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, kPreThreads, smem) != cudaSuccess)
+            return KV_ERR_CUDA;
+        *P_out = std::max(1, occ) * std::max(1, sm_count);
+        return KV_OK;
+    }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kPreThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, fn, *tmap, *c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
 }  // namespace kvp
@@ -64,3 +98,7 @@ int kvp_attn_d64(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArg
                  cudaStream_t st, bool launch, int *P_out);
 int kvp_attn_d128(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sm_count,
                   cudaStream_t st, bool launch, int *P_out);
+int kvp_cascade_d64(int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sm_count,
+                    cudaStream_t st, bool launch, int *P_out);
+int kvp_cascade_d128(int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sm_count,
+                     cudaStream_t st, bool launch, int *P_out);

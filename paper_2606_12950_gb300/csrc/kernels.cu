@@ -1,6 +1,8 @@
 // kernels.cu -- KV append kernel and the launch wrappers of the C ABI
 // (kv_append, kv_workspace_bytes, paged_decode_attn).
+#include <algorithm>
 #include <cmath>
+#include <memory>
 #include <mutex>
 
 #include <cudaTypedefs.h>
@@ -131,6 +133,23 @@ size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
     return hdr + kvp::attn_partial_slots(S, Hkv, P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
 
+// cascade workspace: the above, then the per-sequence skip (padded to 256
+// bytes), then kMaxKeySplits prefix records per (sequence, KV head)
+size_t cascade_ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off, size_t *skip_off, size_t *pre_off)
+{
+    const size_t base = (ws_layout(S, Hkv, G, D, P, part_off) + 255) / 256 * 256;
+    *skip_off = base;
+    *pre_off = base + ((size_t)S * 4 + 255) / 256 * 256;
+    return *pre_off + (size_t)kvp::kMaxKeySplits * S * Hkv * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
+}
+
+int cascade_dispatch(int D, int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sms,
+                     cudaStream_t st, bool launch, int *P_out)
+{
+    if (D == 64) return kvp_cascade_d64(G, tmap, c, grid, sms, st, launch, P_out);
+    return kvp_cascade_d128(G, tmap, c, grid, sms, st, launch, P_out);
+}
+
 }  // namespace
 
 extern "C" {
@@ -174,13 +193,38 @@ int kv_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int max_bloc
     return KV_OK;
 }
 
+int kv_cascade_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int max_blocks, size_t *out_bytes)
+{
+    int G = 0;
+    if (!out_bytes) return KV_ERR_INVALID_ARG;
+    int rc = attn_shape(p, layout, S, Hq, max_blocks, &G);
+    if (rc) return rc;
+    const kv_layout &L = p->desc.layouts[layout];
+    kvp::AttnArgs a{};
+    a.S = S;
+    a.Hkv = L.num_kv_heads;
+    int P = 0;
+    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, 0, p->sm_count, nullptr, false, &P);
+    if (rc) return rc;
+    size_t o1, o2, o3;
+    *out_bytes = cascade_ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &o1, &o2, &o3);
+    return KV_OK;
+}
+
 }  // extern "C"
 
 namespace {
 
+struct CascadePlan {
+    const kv_prefix_group *groups;
+    int n_groups;
+    const int32_t *members;
+};
+
 int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
               uint16_t *out, const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq,
-              float scale, int num_splits, void *workspace, size_t ws_bytes, void *stream)
+              float scale, int num_splits, void *workspace, size_t ws_bytes, void *stream,
+              const CascadePlan *cas = nullptr)
 {
     int G = 0;
     if (num_splits < 0 || !std::isfinite(scale)) return KV_ERR_INVALID_ARG;
@@ -213,11 +257,86 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     rc = dispatch(variant, L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, false, &P);
     if (rc) return rc;
     size_t part_off;
-    const size_t need = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &part_off);
+    if (!cas) {
+        const size_t need = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &part_off);
+        if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
+        a.ws_run = reinterpret_cast<int2 *>(workspace);
+        a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
+        rc = ensure_tmap(p, layout);
+        if (rc) return rc;
+        return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count,
+                        (cudaStream_t)stream, true, &P);
+    }
+
+    // ---- shared-prefix mode: validate the plan, build the prefix kernel's
+    // parameters, then launch prefix kernel, decode kernel and combine ----
+    const int bs = p->desc.block_size, Hkv = L.num_kv_heads;
+    const int ng = cas->n_groups;
+    if (ng < 1 || !cas->groups || !cas->members) return KV_ERR_INVALID_ARG;
+    int64_t nm = 0;
+    for (int i = 0; i < ng; ++i) {
+        const kv_prefix_group &gr = cas->groups[i];
+        if (gr.count < 1 || gr.tokens < kvp::kPreKeys || gr.tokens % kvp::kPreKeys || gr.tokens % bs ||
+            (int64_t)gr.tokens > (int64_t)max_blocks * bs)
+            return KV_ERR_INVALID_ARG;
+        nm += gr.count;
+    }
+    if (nm > S || 2 * (ng + 1) + ng + nm + S > kvp::kCascadeWords) return KV_ERR_INVALID_ARG;
+    auto c = std::make_unique<kvp::CascadeArgs>();
+    int32_t *tile_off = c->data, *mem_off = tile_off + ng + 1, *tokens = mem_off + ng + 1;
+    int32_t *mem = tokens + ng, *skip = mem + nm;
+    std::fill(skip, skip + S, 0);
+    const int MT = kvp::kPreRows / G;
+    int kt_min = INT32_MAX;
+    tile_off[0] = 0;
+    mem_off[0] = 0;
+    for (int i = 0; i < ng; ++i) {
+        const kv_prefix_group &gr = cas->groups[i];
+        tile_off[i + 1] = tile_off[i] + (gr.count + MT - 1) / MT;
+        mem_off[i + 1] = mem_off[i] + gr.count;
+        tokens[i] = gr.tokens;
+        kt_min = std::min(kt_min, gr.tokens / kvp::kPreKeys);
+        for (int j = mem_off[i]; j < mem_off[i + 1]; ++j) {
+            const int32_t s = cas->members[j];
+            if (s < 0 || s >= S || skip[s]) return KV_ERR_INVALID_ARG;  // each sequence in one group at most
+            mem[j] = s;
+            skip[s] = gr.tokens;
+        }
+    }
+    const int tiles = tile_off[ng];
+    size_t skip_off, pre_off;
+    const size_t need = cascade_ws_layout(S, Hkv, G, L.head_dim, P, &part_off, &skip_off, &pre_off);
     if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
-    a.ws_run = reinterpret_cast<int2 *>(workspace);
-    a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
+    uint8_t *ws = reinterpret_cast<uint8_t *>(workspace);
+    c->q = q;
+    c->table = dev_table;
+    c->err = p->desc.device_error;
+    c->ws_pre = reinterpret_cast<float *>(ws + pre_off);
+    c->ws_skip = reinterpret_cast<int32_t *>(ws + skip_off);
+    c->rows_per_page = a.rows_per_page;
+    c->pool_pages = a.pool_pages;
+    c->pages_per_block = a.pages_per_block;
+    c->max_blocks = max_blocks;
+    c->S = S;
+    c->Hkv = Hkv;
+    c->bs = bs;
+    c->n_groups = ng;
+    c->n_members = (int32_t)nm;
+    c->qk_scale = a.qk_scale;
+    int P_pre = 0;
+    rc = cascade_dispatch(L.head_dim, G, nullptr, c.get(), 0, p->sm_count, nullptr, false, &P_pre);
+    if (rc) return rc;
+    // key splits: fill the GPU's CTA slots once, every split non-empty
+    c->KS = std::max(1, std::min({P_pre / std::max(1, tiles * Hkv), kvp::kMaxKeySplits, kt_min}));
+    a.ws_run = reinterpret_cast<int2 *>(ws);
+    a.ws_part = reinterpret_cast<float *>(ws + part_off);
+    a.skip = c->ws_skip;
+    a.ws_pre = c->ws_pre;
+    a.KS = c->KS;
     rc = ensure_tmap(p, layout);
+    if (rc) return rc;
+    rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c.get(), tiles * Hkv * c->KS, p->sm_count,
+                          (cudaStream_t)stream, true, &P_pre);
     if (rc) return rc;
     return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                     true, &P);
@@ -246,3 +365,18 @@ int paged_decode_attn_append(kv_pool *p, int layout, const uint16_t *q, const ui
 }
 
 }  // extern "C"
+
+extern "C" int paged_decode_attn_cascade(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new,
+                                         const uint16_t *v_new, uint16_t *out, const int32_t *dev_table,
+                                         const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq, float scale,
+                                         const kv_prefix_group *groups, int n_groups, const int32_t *members,
+                                         void *workspace, size_t ws_bytes, void *stream)
+{
+    if (n_groups < 0 || (!k_new) != (!v_new)) return KV_ERR_INVALID_ARG;
+    if (n_groups == 0)
+        return attn_call(p, layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale, 0,
+                         workspace, ws_bytes, stream);
+    const CascadePlan plan{groups, n_groups, members};
+    return attn_call(p, layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale, 0,
+                     workspace, ws_bytes, stream, &plan);
+}

@@ -114,6 +114,10 @@ class kv_plan_step(ctypes.Structure):
     ]
 
 
+class kv_prefix_group(ctypes.Structure):
+    _fields_ = [("count", ctypes.c_int32), ("tokens", ctypes.c_int32)]
+
+
 KV_ENGINE_IDLE, KV_ENGINE_SLEEPING, KV_ENGINE_SLEEP_PENDING, KV_ENGINE_ACTIVE, KV_ENGINE_COLD = 0, 1, 2, 3, 4
 KV_ACT_SLEEP, KV_ACT_EVICT, KV_ACT_STOP, KV_ACT_PREEMPT, KV_ACT_ABORT = 1, 2, 3, 4, 5
 
@@ -149,6 +153,8 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
             "paged_decode_attn_append": [P, I, P, P, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "kv_set_attn_variant": [P, I],
+            "kv_cascade_workspace_bytes": [P, I, I, I, I, ctypes.POINTER(SZ)],
+            "paged_decode_attn_cascade": [P, I, P, P, P, P, P, P, I, I, I, F, P, I, P, P, SZ, P],
             "kv_seqtab_create": [P, I, I, I, ctypes.POINTER(P)],
             "kv_seqtab_destroy": [P],
             "kv_seq_reserve": [P, I, I64],
@@ -332,6 +338,40 @@ def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens
            lib().paged_decode_attn_noalloc(pool, layout, _addr(q), _addr(out), _addr(dev_table),
                                            _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq), float(scale),
                                            int(num_splits), _stream(stream)))
+
+
+class PrefixPlan:
+    """Groups of sequences sharing a prefix: [(members, tokens), ...],
+    marshalled once for paged_decode_attn_cascade."""
+
+    def __init__(self, groups):
+        groups = [(list(map(int, m)), int(t)) for m, t in groups]
+        self.n_groups = len(groups)
+        self.groups = (kv_prefix_group * max(1, self.n_groups))()
+        members = [s for m, _ in groups for s in m]
+        self.members = (ctypes.c_int32 * max(1, len(members)))(*members)
+        for i, (m, t) in enumerate(groups):
+            self.groups[i].count = len(m)
+            self.groups[i].tokens = t
+        self.n_members = len(members)
+
+
+def kv_cascade_workspace_bytes(pool, layout: int, S: int, Hq: int, max_blocks: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check("kv_cascade_workspace_bytes", lib().kv_cascade_workspace_bytes(pool, layout, int(S), int(Hq),
+                                                                          int(max_blocks), ctypes.byref(n)))
+    return int(n.value)
+
+
+def paged_decode_attn_cascade(pool, layout: int, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks: int,
+                              S: int, Hq: int, scale: float, plan: PrefixPlan, workspace, ws_bytes: int,
+                              stream=None) -> None:
+    _check("paged_decode_attn_cascade",
+           lib().paged_decode_attn_cascade(pool, layout, _addr(q), _addr(k_new), _addr(v_new), _addr(out),
+                                           _addr(dev_table), _addr(dev_ctx_lens), int(max_blocks), int(S), int(Hq),
+                                           float(scale), ctypes.addressof(plan.groups), plan.n_groups,
+                                           ctypes.addressof(plan.members), _addr(workspace), int(ws_bytes),
+                                           _stream(stream)))
 
 
 def kv_set_attn_variant(pool, variant: int) -> None:

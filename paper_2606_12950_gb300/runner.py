@@ -115,6 +115,16 @@ class DeviceBatch:
                                    self.table, self.lens, self.max_blocks, self.S, self.Hq, self.b.scale,
                                    self.num_splits, self.ws, self.ws.numel(), stream)
 
+    def cascade(self, plan, fused: bool = True, stream=None) -> None:
+        """Shared-prefix attention (with the fused append unless fused=False)."""
+        need = K.kv_cascade_workspace_bytes(self.pool.handle, self.layout, self.S, self.Hq, self.max_blocks)
+        if need > self.ws.numel():
+            self.ws = torch.zeros(need, dtype=torch.uint8, device=self.pool.device)
+        K.paged_decode_attn_cascade(self.pool.handle, self.layout, self.q, self.k_new if fused else None,
+                                    self.v_new if fused else None, self.out, self.table, self.lens,
+                                    self.max_blocks, self.S, self.Hq, self.b.scale, plan, self.ws,
+                                    self.ws.numel(), stream)
+
     def out_f64(self) -> np.ndarray:
         return self.out.float().cpu().numpy().astype(np.float64)
 
@@ -157,3 +167,15 @@ class DeviceSteps:
         K.paged_decode_attn(self.pool.handle, self.layout, self.q, self.out, self.table, self.lens,
                             self.max_blocks, self.S, self.Hq, self.scale, self.num_splits, self.ws,
                             self.ws.numel(), stream)
+
+    def use_cascade(self) -> None:
+        """Size the workspace for paged_decode_attn_cascade."""
+        need = K.kv_cascade_workspace_bytes(self.pool.handle, self.layout, self.S, self.Hq, self.max_blocks)
+        if need > self.ws.numel():
+            self.ws = torch.empty(need, dtype=torch.uint8, device=self.pool.device)
+
+    def cascade(self, plan, fused: bool = True, stream=None) -> None:
+        K.paged_decode_attn_cascade(self.pool.handle, self.layout, self.q, self.k_new if fused else None,
+                                    self.v_new if fused else None, self.out, self.table, self.lens,
+                                    self.max_blocks, self.S, self.Hq, self.scale, plan, self.ws,
+                                    self.ws.numel(), stream)

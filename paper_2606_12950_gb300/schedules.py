@@ -89,6 +89,13 @@ class AgentChains:
         self.ctx += 1
         self.left -= 1
 
+    def prefix_plan(self) -> "K.PrefixPlan":
+        """Every chain holds the system prompt's blocks at the start of its
+        table: one shared-prefix group over all decode rows."""
+        if getattr(self, "_plan", None) is None:
+            self._plan = K.PrefixPlan([(range(self.n), self.prefix_tokens)])
+        return self._plan
+
     def close(self) -> None:
         self.tab.close()
 

@@ -134,6 +134,21 @@ class Batch:
         return 2 * self.Hkv * self.bs * self.d
 
 
+def share_prefix(b: "Batch", groups) -> "Batch":
+    """Make each group's members hold their first ``tokens`` tokens in the same
+    physical blocks as the group's first member (a prefix shared by
+    reference); ``groups`` = [(members, tokens), ...], tokens a multiple of
+    the block size.  The members' own blocks for those positions become
+    unused.  Returns ``b`` with its table changed in place."""
+    for members, tokens in groups:
+        assert tokens % b.bs == 0
+        nb = tokens // b.bs
+        lead = int(members[0])
+        for s in members[1:]:
+            b.table[int(s), :nb] = b.table[lead, :nb]
+    return b
+
+
 def make_batch(
     seed: int,
     pre_lens,

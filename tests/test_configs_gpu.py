@@ -40,11 +40,18 @@ class Runner:
         self.table = torch.full((rows, max_blocks), -1, dtype=torch.int32, device="cuda")
         self.lens = torch.zeros(rows, dtype=torch.int32, device="cuda")
 
-    def step(self, tab, S, step):
+    def step(self, tab, S, step, plan=None):
         q, kn, vn = W.step_rows(self.seed, step, S, self.Hq, self.Hkv, self.d)
         qd, kd, vd = _dev_bits(q), _dev_bits(kn), _dev_bits(vn)
         out = torch.empty_like(qd)
         tab.sync(self.table, self.lens)
+        if plan is not None:  # shared-prefix attention with the fused append
+            nbytes = K.kv_cascade_workspace_bytes(self.pool.handle, self.layout, S, self.Hq, self.max_blocks)
+            ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+            K.paged_decode_attn_cascade(self.pool.handle, self.layout, qd, kd, vd, out, self.table, self.lens,
+                                        self.max_blocks, S, self.Hq, self.scale, plan, ws, nbytes)
+            torch.cuda.synchronize()
+            return q, kn, vn, out.float().cpu().numpy().astype(np.float64)
         K.kv_append(self.pool.handle, self.layout, kd, vd, self.table, self.lens, self.max_blocks, S)
         nbytes = K.kv_workspace_bytes(self.pool.handle, self.layout, S, self.Hq, self.max_blocks)
         ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
@@ -67,7 +74,7 @@ def _sample(rng, lens, k):
     return np.array(sorted(pick), np.int32)
 
 
-def _run_chains(n_chains, steps, median, max_out, sample, seed=1003, check_every=1):
+def _run_chains(n_chains, steps, median, max_out, sample, seed=1003, check_every=1, cascade=False):
     from paper_2606_12950_gb300.runner import DevicePool
     from paper_2606_12950_gb300.schedules import AgentChains
 
@@ -84,7 +91,7 @@ def _run_chains(n_chains, steps, median, max_out, sample, seed=1003, check_every
     rng = np.random.default_rng(seed + 5)
     for step in range(steps):
         ch.step()
-        q, kn, vn, got = run.step(ch.tab, n_chains, step)
+        q, kn, vn, got = run.step(ch.tab, n_chains, step, plan=ch.prefix_plan() if cascade else None)
         table, lens = ch.tab.host()
         table, lens = table[:n_chains], lens[:n_chains]
         oracle.append(host_pool, n_pages, page_elems, bs, Hkv, d, kn, vn, table, lens, inplace=True)
@@ -105,6 +112,18 @@ def test_agent_chains_full_size():
     """256 concurrent chains, 2048-token shared prefix, stage outputs
     lognormal(300), reservations true x U[0.8, 1.5]."""
     _run_chains(256, steps=3, median=300.0, max_out=4096, sample=16)
+
+
+def test_agent_chains_full_size_cascade():
+    """The same 256 chains through shared-prefix attention: the 2048-token
+    prompt is attended once per KV head for all chains, each chain's own
+    context streamed and merged."""
+    _run_chains(256, steps=3, median=300.0, max_out=4096, sample=16, cascade=True)
+
+
+def test_agent_chains_stage_turnover_cascade():
+    ends, done, misses = _run_chains(48, steps=40, median=5.0, max_out=40, sample=0, check_every=4, cascade=True)
+    assert ends > 48 and done > 0 and misses > 0
 
 
 def test_agent_chains_stage_turnover():
