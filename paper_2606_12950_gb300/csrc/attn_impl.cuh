@@ -752,13 +752,14 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
 }
 
 // ------------------------------------------------------------ combine ---
-// Split-K combine: for each (sequence, KV head) run cut by part boundaries,
-// merge its parts' partials (m_k, l_k, o_k) in part order:
+// Split-K combine: for each (sequence, KV head) run cut by part boundaries
+// (or with a shared prefix), merge its records (m_k, l_k, o_k) in order:
 //     M = max_k m_k,  out = sum_k 2^(m_k - M) o_k / sum_k 2^(m_k - M) l_k
-// (base-2 online-softmax state).  One CTA per run; runs finished inside the
+// (base-2 online-softmax state).  One CTA per run, covering all G*D output
+// columns: NG thread groups of G*D/4 threads (one float4 column each) take
+// records k = grp, grp + NG, ..., then merge their states in group order, so
+// the result depends only on the run's shape.  Runs finished inside the
 // attention kernel return at once.
-constexpr int kCombineThreads = 256;
-
 struct CombineArgs {
     uint16_t *out;
     const int2 *ws_run;    // per run: (first part, parts), parts = 0 when not split
@@ -770,27 +771,22 @@ struct CombineArgs {
     int32_t KS;
 };
 
-// columns (float4 of o) per combine CTA, and CTAs per run
 template <int D, int G>
-__host__ __device__ constexpr int combine_cols()
-{
-    return G * D / 4 < 32 ? G * D / 4 : ((G * D / 4) % 32 == 0 ? 32 : 16);
-}
+__host__ __device__ constexpr int combine_groups() { return (G * D / 4) >= 256 ? 1 : 256 / (G * D / 4); }
 template <int D, int G>
-__host__ __device__ constexpr int combine_ctas_per_run() { return (G * D / 4) / combine_cols<D, G>(); }
+__host__ __device__ constexpr int combine_threads() { return (G * D / 4) * combine_groups<D, G>(); }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_constant__ CombineArgs c)
+__global__ void __launch_bounds__(combine_threads<D, G>()) combine_kernel(const __grid_constant__ CombineArgs c)
 {
     constexpr uint32_t MF = merge_floats<D, G>();
-    constexpr int CW = combine_cols<D, G>();       // columns of this CTA
-    constexpr int CB = combine_ctas_per_run<D, G>();
-    constexpr int NSPLIT = kCombineThreads / CW;   // thread groups splitting the partials
-    static_assert(CW * CB == G * D / 4, "columns must tile the output");
-    __shared__ float s_M[kCombineThreads];
-    __shared__ float s_L[kCombineThreads];
-    __shared__ float4 s_O[kCombineThreads];
-    const int r = blockIdx.x / CB, cb = blockIdx.x % CB;
+    constexpr int NC = G * D / 4;  // float4 columns of a run's output
+    constexpr int NG = combine_groups<D, G>();
+    constexpr int T = NC * NG;
+    __shared__ float s_M[NG > 1 ? T : 1];
+    __shared__ float s_L[NG > 1 ? T : 1];
+    __shared__ float4 s_O[NG > 1 ? T : 1];
+    const int r = blockIdx.x;
     grid_dependency_wait();  // the attention grid's partials and run table
     const int2 info = c.ws_run[r];
     const int s = r / c.Hkv, g = r % c.Hkv;
@@ -800,15 +796,14 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
     const float *base = c.ws_part + ((int64_t)r + info.x) * MF;
     uint16_t *orow = c.out + ((int64_t)s * c.Hkv * G + (int64_t)g * G) * D;
     const int tid = threadIdx.x;
-    const int col = cb * CW + tid % CW;
-    const int grp = tid / CW;
+    const int col = tid % NC;
+    const int grp = tid / NC;
     const int h = (col * 4) / D;
-    // online merge of this group's partials (k = grp, grp + NSPLIT, ...):
-    // M running max, L and O relative to M
+    // online merge of this group's records: M running max, L and O relative to M
     float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-    for (int k = grp; k < cnt; k += NSPLIT) {
+#pragma unroll 4
+    for (int k = grp; k < cnt; k += NG) {
         const float *sl = k < npre ? c.ws_pre + (((int64_t)k * c.S + s) * c.Hkv + g) * MF
                                    : base + (int64_t)(k - npre) * MF;
         const float mk = sl[G * D + h];
@@ -823,32 +818,33 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const __grid_c
         O.w = O.w * sa + ok.w * sb;
         M = Mn;
     }
-    s_M[tid] = M;
-    s_L[tid] = L;
-    s_O[tid] = O;
-    __syncthreads();
-    if (grp == 0) {
-        // merge the groups in order, so the result depends only on the run's shape
-        for (int j = 1; j < NSPLIT; ++j) {
-            const float mj = s_M[tid + j * CW];
-            if (mj == -INFINITY) continue;  // group had no partials
+    if constexpr (NG > 1) {
+        s_M[tid] = M;
+        s_L[tid] = L;
+        s_O[tid] = O;
+        __syncthreads();
+        if (grp != 0) return;
+        // merge the groups in order
+        for (int j = 1; j < NG; ++j) {
+            const float mj = s_M[tid + j * NC];
+            if (mj == -INFINITY) continue;  // group had no records
             const float Mn = fmaxf(M, mj);
             const float sa = fast_exp2(M - Mn), sb = fast_exp2(mj - Mn);
-            const float4 oj = s_O[tid + j * CW];
-            L = L * sa + s_L[tid + j * CW] * sb;
+            const float4 oj = s_O[tid + j * NC];
+            L = L * sa + s_L[tid + j * NC] * sb;
             O.x = O.x * sa + oj.x * sb;
             O.y = O.y * sa + oj.y * sb;
             O.z = O.z * sa + oj.z * sb;
             O.w = O.w * sa + oj.w * sb;
             M = Mn;
         }
-        __nv_bfloat162 lo = __floats2bfloat162_rn(O.x / L, O.y / L);
-        __nv_bfloat162 hi = __floats2bfloat162_rn(O.z / L, O.w / L);
-        uint2 w2;
-        w2.x = *reinterpret_cast<uint32_t *>(&lo);
-        w2.y = *reinterpret_cast<uint32_t *>(&hi);
-        *reinterpret_cast<uint2 *>(orow + col * 4) = w2;
     }
+    __nv_bfloat162 lo = __floats2bfloat162_rn(O.x / L, O.y / L);
+    __nv_bfloat162 hi = __floats2bfloat162_rn(O.z / L, O.w / L);
+    uint2 w2;
+    w2.x = *reinterpret_cast<uint32_t *>(&lo);
+    w2.y = *reinterpret_cast<uint32_t *>(&hi);
+    *reinterpret_cast<uint2 *>(orow + col * 4) = w2;
 }
 
 // host helpers ---------------------------------------------------------------

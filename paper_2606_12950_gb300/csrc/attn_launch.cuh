@@ -50,8 +50,8 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
     CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv, a.skip, a.ws_pre, a.KS};
     cudaLaunchConfig_t ccfg = cfg;
-    ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv * combine_ctas_per_run<D, G>()));
-    ccfg.blockDim = dim3(kCombineThreads);
+    ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv));
+    ccfg.blockDim = dim3(combine_threads<D, G>());
     ccfg.dynamicSmemBytes = 0;
     if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G>, c) != cudaSuccess) return KV_ERR_CUDA;
     return KV_OK;
