@@ -104,6 +104,23 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def aggregate_ranks(dist, device, ms: float, e2e_ms: float, units: dict) -> tuple:
+    """Whole-job figures of N independent replicas: the slowest rank's time
+    (max over ranks) and the units every rank processed (sum over ranks).
+    With dist None (one process) the inputs come back unchanged."""
+    if dist is None:
+        return ms, e2e_ms, dict(units)
+    import torch
+
+    keys = sorted(units)
+    t = torch.tensor([ms, e2e_ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    u = torch.tensor([float(units[k]) for k in keys], dtype=torch.float64, device=device)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    tl, ul = t.tolist(), u.tolist()
+    return tl[0], tl[1], dict(zip(keys, ul))
+
+
 def oracle_baseline(b, budget_s: float):
     """Time the fp64 C oracle (single thread) on whole decode steps of the
     same workload (append + attention over every sequence) until budget_s
@@ -421,18 +438,12 @@ def main():
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
     attn_ms = [a.elapsed_time(z) for a, z in evs]
-    if dist:
-        tt = torch.tensor([ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
     err = wl.pool.error(stream)
 
-    dram_total = sum(x[0] for x in step_bytes)
-    logical_total = sum(x[1] for x in step_bytes)
-    gbs = dram_total / (ms * 1e-3) / 1e9 * world
-    tokens_per_s = wl.S * args.steps / (ms * 1e-3) * world
+    dram_rank = sum(x[0] for x in step_bytes)
+    logical_rank = sum(x[1] for x in step_bytes)
     attn_avg_ms = float(np.mean(attn_ms))
-    attn_gbs = dram_total / args.steps / (attn_avg_ms * 1e-3) / 1e9
+    attn_gbs = dram_rank / args.steps / (attn_avg_ms * 1e-3) / 1e9  # this rank's kernels
     peak, peak_kind = load_peaks()
 
     # end to end: q / k / v from pinned host memory, output back to host, every step
@@ -467,7 +478,12 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    e2e_gbs = e2e_bytes / (e2e_ms * 1e-3) / 1e9 * world
+    ms, e2e_ms, tot = aggregate_ranks(dist, torch.device("cuda", local), ms, e2e_ms,
+                                      {"dram": dram_rank, "logical": logical_rank, "tokens": wl.S * args.steps,
+                                       "e2e": e2e_bytes})
+    gbs = tot["dram"] / (ms * 1e-3) / 1e9
+    tokens_per_s = tot["tokens"] / (ms * 1e-3)
+    e2e_gbs = tot["e2e"] / (e2e_ms * 1e-3) / 1e9
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and args.workload == "llama8b":
@@ -507,8 +523,8 @@ def main():
         "device_error": err,
         "cpu_baseline": cpu,
     }
-    if logical_total != dram_total:
-        line["logical_gbs"] = logical_total / (ms * 1e-3) / 1e9 * world
+    if tot["logical"] != tot["dram"]:
+        line["logical_gbs"] = tot["logical"] / (ms * 1e-3) / 1e9
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:

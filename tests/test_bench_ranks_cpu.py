@@ -1,0 +1,75 @@
+"""The benchmark's multi-rank path on the CPU: two gloo ranks, each a
+replica with its own work, reduce to the whole-job figures (the slowest
+rank's time, the sum of the units), and the reference arm prints on rank 0
+only."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+torch = pytest.importorskip("torch")
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank(rank, world, port, out):
+    import torch.distributed as dist
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    # rank r: 10 + r ms, bytes 100 * (r + 1), tokens 64 each
+    got = bench.aggregate_ranks(dist, torch.device("cpu"), 10.0 + rank, 20.0 - rank,
+                                {"dram": 100.0 * (rank + 1), "tokens": 64.0})
+    with open(os.path.join(out, f"rank{rank}.json"), "w") as f:
+        json.dump(got, f)
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_aggregate_over_two_gloo_ranks(tmp_path):
+    import torch.multiprocessing as mp
+
+    port = _free_port()
+    mp.start_processes(_rank, args=(2, port, str(tmp_path)), nprocs=2, join=True, start_method="spawn")
+    for r in range(2):
+        ms, e2e_ms, units = json.load(open(tmp_path / f"rank{r}.json"))
+        assert ms == 11.0 and e2e_ms == 20.0  # the slowest rank's times
+        assert units == {"dram": 300.0, "tokens": 128.0}  # every rank's units
+
+
+def test_single_process_passes_through():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    assert bench.aggregate_ranks(None, None, 3.0, 4.0, {"a": 5}) == (3.0, 4.0, {"a": 5})
+
+
+def test_reference_arm_prints_on_rank0_only():
+    """Under torchrun only rank 0 runs and prints the oracle's line; rank 1
+    exits 0 without work (here: two ranks launched by hand, no rendezvous
+    needed because the reference arm makes none)."""
+    env = dict(os.environ, WORLD_SIZE="2", RANK="1", LOCAL_RANK="1")
+    r1 = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                         "--warmup", "0", "--gpus", "2"], env=env, capture_output=True, text=True, timeout=300)
+    assert r1.returncode == 0 and r1.stdout.strip() == ""
+    env.update(RANK="0", LOCAL_RANK="0")
+    r0 = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                         "--warmup", "0", "--gpus", "2"], env=env, capture_output=True, text=True, timeout=600)
+    assert r0.returncode == 0, r0.stderr[-2000:]
+    lines = [l for l in r0.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["cpu_baseline"]["kind"] == "oracle"
