@@ -193,8 +193,17 @@ class Llama8B:
         total = 2 * (args.warmup + args.steps) + 8
         b = W.config2_llama8b(steps=max(100, total))
         self.b = b
-        self.pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)], shuffle_seed=b.meta["seed"])
-        self.pool.upload(b.pool)
+        vmm = getattr(args, "pool", "fixed") == "vmm"
+        if vmm:
+            # elastic pool: 4x the batch's need reserved as virtual memory,
+            # chunks mapped as the reservations below allocate blocks
+            from paper_2606_12950_gb300.runner import VmmPool
+
+            self.pool = VmmPool(4 * b.n_pages * b.page_elems * 2, b.page_elems * 2, b.bs, [(b.Hkv, b.d)],
+                                shuffle_seed=b.meta["seed"])
+        else:
+            self.pool = DevicePool(b.n_pages, b.page_elems * 2, b.bs, [(b.Hkv, b.d)], shuffle_seed=b.meta["seed"])
+            self.pool.upload(b.pool)
         if args.variant:
             self.pool.set_variant(args.variant)
         self.tab = K.SeqTab(self.pool.handle, 0, b.S, b.max_blocks)
@@ -202,6 +211,9 @@ class Llama8B:
         for s in range(b.S):
             self.tab.reserve(s, int(self.pre[s]) + total)
             self.tab.set_len(s, int(self.pre[s]))
+        if vmm:
+            table, _ = self.tab.host()
+            self.pool.fill_random(np.unique(table[table >= 0]), b.meta["seed"])
         self.bufs = [DeviceSteps(self.pool, 0, b.S, b.S, b.Hq, b.Hkv, b.d, b.max_blocks, b.scale, b.q, b.k_new,
                                  b.v_new, args.num_splits)]
         self.S = b.S
@@ -352,6 +364,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
+    ap.add_argument("--pool", default="fixed", choices=["fixed", "vmm"],
+                    help="llama8b: a fixed device buffer, or the VMM-backed elastic pool")
     ap.add_argument("--no-cascade", action="store_true",
                     help="agent chains: stream the shared prefix per chain instead of once per KV head")
     args = ap.parse_args()
@@ -503,6 +517,7 @@ def main():
             traffic = None
 
     config = {"workload": wl.name, **wl.config, "num_splits": args.num_splits, "variant": args.variant,
+              "pool": args.pool if args.workload == "llama8b" else "fixed",
               "append": "separate kernel" if args.separate_append else "fused into attention",
               "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
                                 else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,

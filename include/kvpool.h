@@ -102,6 +102,7 @@ typedef struct kv_stats {
     int64_t blocks_capacity[KV_MAX_LAYOUTS]; /* used + cached + unassigned/k */
     uint64_t bytes_used;                     /* sum of used blocks' bytes */
     uint64_t bytes_total;                    /* pages_total * page_bytes */
+    uint64_t bytes_mapped;                   /* physically backed bytes (VMM pool); bytes_total otherwise */
 } kv_stats;
 
 /* ---------------------------------------------------------------- pool --- */
@@ -118,8 +119,69 @@ typedef struct kv_stats {
  */
 int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool);
 
-/* Release host metadata.  The device buffer is the caller's. */
+/* Release host metadata.  The device buffer of a fixed pool is the caller's;
+ * a VMM pool's mappings and reserved range are released (after a device
+ * synchronize when the library's CUDA backend owns them). */
 int kv_pool_destroy(kv_pool *pool);
+
+/*
+ * VMM-backed elastic pool (§III-C, spatial multiplexing with a virtual-memory
+ * KV cache).  The pool's pool_bytes are a reserved virtual range that may
+ * exceed the physical memory the KV may use (overcommitment, Table 5); it is
+ * cut into chunks of chunk_bytes (a multiple of the superpage, so superpages
+ * never straddle chunks) that are physically mapped when kv_alloc_blocks
+ * needs their superpages, and unmapped by kv_pool_trim.  kv_alloc_blocks maps
+ * first and allocates after, all-or-nothing: a chunk that cannot be mapped
+ * (device memory exhausted, physical_limit or the shared budget reached)
+ * rejects the request with KV_ERR_OUT_OF_BLOCKS and allocates nothing.
+ *
+ * Backends:
+ *   map_fn == NULL: CUDA virtual memory management on `device`.  The library
+ *     reserves the range (desc->device_base must be NULL; read it back with
+ *     kv_pool_get_base), chunk_bytes 0 = the allocation granularity (else a
+ *     multiple of it), and backs every unmapped chunk with one shared guard
+ *     allocation, so a device table entry naming an unallocated block reads
+ *     zeros or stale data instead of faulting.
+ *   map_fn != NULL: the caller's backing over its own range desc->device_base
+ *     (e.g. a framework's allocator, or a host fake in tests): the library
+ *     calls map_fn(ctx, offset, bytes) / unmap_fn(ctx, offset, bytes) per
+ *     chunk (0 = success) and chunk_bytes must be given.
+ * The pool covers whole chunks (pool_bytes is rounded down).  Block tables
+ * uploaded with kv_block_table_upload may name only blocks in mapped chunks.
+ * Errors: KV_ERR_INVALID_ARG, KV_ERR_CUDA (reservation or guard mapping).
+ */
+typedef struct kv_budget kv_budget;
+
+typedef struct kv_vmm_desc {
+    uint64_t chunk_bytes;     /* mapping unit; 0 = granularity (CUDA backend only) */
+    uint64_t physical_limit;  /* at most this many bytes mapped in this pool; 0 = no limit */
+    kv_budget *budget;        /* optional limit shared by several pools (mapped bytes of all of them) */
+    int32_t device;           /* CUDA device ordinal (CUDA backend) */
+    int32_t reserved;
+    int (*map_fn)(void *ctx, uint64_t offset, uint64_t bytes);
+    int (*unmap_fn)(void *ctx, uint64_t offset, uint64_t bytes);
+    void *ctx;
+} kv_vmm_desc;
+
+int kv_pool_create_vmm(const kv_pool_desc *desc, const kv_vmm_desc *vmm, kv_pool **out_pool);
+
+/* Device address of the pool's first byte (the reserved range of a VMM pool). */
+int kv_pool_get_base(const kv_pool *pool, void **base);
+
+/*
+ * Give memory back: superpages whose blocks are all free return from their
+ * layout's free list to the shared list (so other layouts can use them), and
+ * a VMM pool unmaps every chunk whose superpages are all free, adding the
+ * bytes to *released_bytes (may be NULL).  The CUDA backend synchronises the
+ * device before unmapping (kernels in flight may still read freed blocks).
+ */
+int kv_pool_trim(kv_pool *pool, uint64_t *released_bytes);
+
+/* A physical-memory budget shared by VMM pools (e.g. M_total - M_res of the
+ * node, §III-C).  Destroy it after every pool that uses it. */
+int kv_budget_create(uint64_t limit_bytes, kv_budget **out);
+int kv_budget_destroy(kv_budget *budget);
+int kv_budget_used(const kv_budget *budget, uint64_t *used_bytes);
 
 /*
  * Reserve n blocks of layout `layout` (Eq. 2's per-stage reservation is n =

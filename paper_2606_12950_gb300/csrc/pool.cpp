@@ -37,6 +37,7 @@ bool carve(kv_pool *p, int layout)
     if (p->super_free.empty()) return false;
     int32_t sp = p->super_free.back();
     p->super_free.pop_back();
+    if (p->vmm.active) p->vmm.free_supers[(size_t)(sp / p->vmm.supers_per_chunk)] -= 1;
     int32_t k = p->pages_per_block[layout];
     int32_t nb = p->super_pages / k;
     int64_t first = (int64_t)sp * p->super_pages;
@@ -118,6 +119,7 @@ int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool)
 int kv_pool_destroy(kv_pool *pool)
 {
     if (!pool) return KV_ERR_INVALID_ARG;
+    if (pool->vmm.active) kvp_vmm_release_all(pool);
     delete pool;
     return KV_OK;
 }
@@ -127,10 +129,19 @@ int kv_alloc_blocks(kv_pool *p, int layout, int n, int32_t *out_ids)
     if (!layout_ok(p, layout) || n < 0 || (n > 0 && !out_ids)) return KV_ERR_INVALID_ARG;
     std::lock_guard<std::mutex> g(p->mu);
     int32_t k = p->pages_per_block[layout];
-    // capacity check first so the call is all-or-nothing
-    int64_t avail = (int64_t)p->free_blocks[layout].size() +
-                    (int64_t)p->super_free.size() * (p->super_pages / k);
-    if (avail < n) return KV_ERR_OUT_OF_BLOCKS;
+    // capacity check first so the call is all-or-nothing; a VMM pool maps the
+    // chunks it lacks before anything is allocated (a chunk that cannot be
+    // mapped rejects the request; chunks mapped so far stay as free capacity)
+    const int64_t per_super = p->super_pages / k;
+    int64_t avail = (int64_t)p->free_blocks[layout].size() + (int64_t)p->super_free.size() * per_super;
+    if (avail < n) {
+        if (!p->vmm.active) return KV_ERR_OUT_OF_BLOCKS;
+        const int64_t supers = (n - avail + per_super - 1) / per_super;
+        const int64_t chunks = (supers + p->vmm.supers_per_chunk - 1) / p->vmm.supers_per_chunk;
+        if (chunks > (int64_t)p->vmm.unmapped_order.size()) return KV_ERR_OUT_OF_BLOCKS;
+        for (int64_t c = 0; c < chunks; ++c)
+            if (kvp_vmm_map_chunk(p) != KV_OK) return KV_ERR_OUT_OF_BLOCKS;
+    }
     for (int i = 0; i < n; ++i) {
         if (p->free_blocks[layout].empty()) carve(p, layout);
         int32_t id = p->free_blocks[layout].back();
@@ -201,15 +212,76 @@ int kv_pool_stats(const kv_pool *p, kv_stats *out)
     kv_pool *mp = const_cast<kv_pool *>(p);
     std::lock_guard<std::mutex> g(mp->mu);
     out->pages_total = p->n_pages;
-    out->pages_unassigned = (int64_t)p->super_free.size() * p->super_pages;
+    const int64_t unmapped_supers =
+        p->vmm.active ? (int64_t)p->vmm.unmapped_order.size() * p->vmm.supers_per_chunk : 0;
+    out->pages_unassigned = ((int64_t)p->super_free.size() + unmapped_supers) * p->super_pages;
     out->bytes_total = (uint64_t)p->n_pages * p->page_bytes;
     for (int l = 0; l < p->desc.num_layouts; ++l) {
         out->blocks_used[l] = p->used_blocks[l];
         out->blocks_cached[l] = (int64_t)p->free_blocks[l].size();
         out->blocks_capacity[l] = p->used_blocks[l] + out->blocks_cached[l] +
-                                  (int64_t)p->super_free.size() * (p->super_pages / p->pages_per_block[l]);
+                                  ((int64_t)p->super_free.size() + unmapped_supers) *
+                                      (p->super_pages / p->pages_per_block[l]);
         out->bytes_used += (uint64_t)p->used_blocks[l] * p->block_bytes[l];
     }
+    out->bytes_mapped = p->vmm.active ? p->vmm.mapped_bytes : out->bytes_total;
+    return KV_OK;
+}
+
+int kv_pool_trim(kv_pool *p, uint64_t *released_bytes)
+{
+    if (!p) return KV_ERR_INVALID_ARG;
+    std::lock_guard<std::mutex> g(p->mu);
+    // 1. superpages whose blocks are all free in their layout's list go back
+    //    to the shared free list (any layout may carve them again)
+    const int64_t K = p->super_pages;
+    for (int l = 0; l < p->desc.num_layouts; ++l) {
+        auto &fl = p->free_blocks[l];
+        if (fl.empty()) continue;
+        const int32_t per_super = (int32_t)(K / p->pages_per_block[l]);
+        std::unordered_map<int32_t, int32_t> cnt;
+        for (int32_t id : fl) cnt[(int32_t)(id / K)] += 1;
+        std::vector<int32_t> whole;
+        for (auto &kv : cnt)
+            if (kv.second == per_super) whole.push_back(kv.first);
+        if (whole.empty()) continue;
+        std::sort(whole.begin(), whole.end());
+        std::vector<int32_t> keep;
+        keep.reserve(fl.size());
+        for (int32_t id : fl)
+            if (!std::binary_search(whole.begin(), whole.end(), (int32_t)(id / K))) keep.push_back(id);
+        fl.swap(keep);
+        p->carved_blocks[l] -= (int64_t)whole.size() * per_super;
+        for (auto it = whole.rbegin(); it != whole.rend(); ++it) {
+            p->super_free.push_back(*it);
+            if (p->vmm.active) p->vmm.free_supers[(size_t)(*it / p->vmm.supers_per_chunk)] += 1;
+        }
+    }
+    // 2. a VMM pool unmaps every chunk whose superpages are all free
+    uint64_t released = 0;
+    if (p->vmm.active) {
+        const int32_t spc = p->vmm.supers_per_chunk;
+        std::vector<int64_t> chunks;
+        for (int64_t c = 0; c < p->vmm.n_chunks; ++c)
+            if (p->vmm.mapped[(size_t)c] && p->vmm.free_supers[(size_t)c] == spc) chunks.push_back(c);
+        if (!chunks.empty()) {
+            // kernels still in flight may read blocks freed on the host
+            if (!p->vmm.map_fn && cudaDeviceSynchronize() != cudaSuccess) return KV_ERR_CUDA;
+            std::vector<int32_t> keep;
+            keep.reserve(p->super_free.size());
+            for (int32_t sp : p->super_free) {
+                const int64_t c = sp / spc;
+                if (!std::binary_search(chunks.begin(), chunks.end(), c)) keep.push_back(sp);
+            }
+            p->super_free.swap(keep);
+            for (int64_t c : chunks) {
+                const int rc = kvp_vmm_unmap_chunk(p, c);
+                if (rc) return rc;
+                released += p->vmm.chunk_bytes;
+            }
+        }
+    }
+    if (released_bytes) *released_bytes = released;
     return KV_OK;
 }
 

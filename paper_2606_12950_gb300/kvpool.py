@@ -75,6 +75,23 @@ class kv_stats(ctypes.Structure):
         ("blocks_capacity", ctypes.c_int64 * KV_MAX_LAYOUTS),
         ("bytes_used", ctypes.c_uint64),
         ("bytes_total", ctypes.c_uint64),
+        ("bytes_mapped", ctypes.c_uint64),
+    ]
+
+
+MAP_FN = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint64)
+
+
+class kv_vmm_desc(ctypes.Structure):
+    _fields_ = [
+        ("chunk_bytes", ctypes.c_uint64),
+        ("physical_limit", ctypes.c_uint64),
+        ("budget", ctypes.c_void_p),
+        ("device", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+        ("map_fn", MAP_FN),
+        ("unmap_fn", MAP_FN),
+        ("ctx", ctypes.c_void_p),
     ]
 
 
@@ -154,6 +171,12 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn_append": [P, I, P, P, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "kv_set_attn_variant": [P, I],
             "kv_cascade_workspace_bytes": [P, I, I, I, I, ctypes.POINTER(SZ)],
+            "kv_pool_create_vmm": [ctypes.POINTER(kv_pool_desc), ctypes.POINTER(kv_vmm_desc), ctypes.POINTER(P)],
+            "kv_pool_get_base": [P, ctypes.POINTER(P)],
+            "kv_pool_trim": [P, ctypes.POINTER(U64)],
+            "kv_budget_create": [U64, ctypes.POINTER(P)],
+            "kv_budget_destroy": [P],
+            "kv_budget_used": [P, ctypes.POINTER(U64)],
             "paged_decode_attn_cascade": [P, I, P, P, P, P, P, P, I, I, I, F, P, I, P, P, SZ, P],
             "kv_seqtab_create": [P, I, I, I, ctypes.POINTER(P)],
             "kv_seqtab_destroy": [P],
@@ -230,8 +253,74 @@ def kv_pool_create(device_base, pool_bytes: int, block_size: int, layouts, devic
     return h.value
 
 
+def kv_pool_create_vmm(pool_bytes: int, block_size: int, layouts, device_error, page_bytes: int = 0,
+                       shuffle_seed: int = 0, chunk_bytes: int = 0, physical_limit: int = 0, budget=None,
+                       device: int = 0, backend=None, device_base=None):
+    """A VMM-backed pool.  backend=None: CUDA VMM (the library reserves the
+    range); else an object with map(offset, bytes) / unmap(offset, bytes)
+    returning 0 on success, over the caller's range device_base."""
+    d = kv_pool_desc()
+    d.device_base = device_base
+    d.pool_bytes = int(pool_bytes)
+    d.block_size = int(block_size)
+    d.num_layouts = len(layouts)
+    for i, (h, hd) in enumerate(layouts):
+        d.layouts[i].num_kv_heads = int(h)
+        d.layouts[i].head_dim = int(hd)
+    d.page_bytes = int(page_bytes)
+    d.device_error = _addr(device_error)
+    d.shuffle_seed = int(shuffle_seed)
+    v = kv_vmm_desc()
+    v.chunk_bytes = int(chunk_bytes)
+    v.physical_limit = int(physical_limit)
+    v.budget = budget
+    v.device = int(device)
+    keep = None
+    if backend is not None:
+        keep = (MAP_FN(lambda ctx, off, n: int(backend.map(int(off), int(n)))),
+                MAP_FN(lambda ctx, off, n: int(backend.unmap(int(off), int(n)))))
+        v.map_fn, v.unmap_fn = keep
+    out = ctypes.c_void_p()
+    _check("kv_pool_create_vmm", lib().kv_pool_create_vmm(ctypes.byref(d), ctypes.byref(v), ctypes.byref(out)))
+    if keep is not None:
+        _callbacks[out.value] = keep  # the library keeps calling them until destroy
+    return out.value
+
+
+_callbacks = {}
+
+
+def kv_pool_get_base(pool) -> int:
+    b = ctypes.c_void_p()
+    _check("kv_pool_get_base", lib().kv_pool_get_base(pool, ctypes.byref(b)))
+    return int(b.value or 0)
+
+
+def kv_pool_trim(pool) -> int:
+    r = ctypes.c_uint64(0)
+    _check("kv_pool_trim", lib().kv_pool_trim(pool, ctypes.byref(r)))
+    return int(r.value)
+
+
+def kv_budget_create(limit_bytes: int):
+    out = ctypes.c_void_p()
+    _check("kv_budget_create", lib().kv_budget_create(int(limit_bytes), ctypes.byref(out)))
+    return out.value
+
+
+def kv_budget_destroy(budget) -> None:
+    _check("kv_budget_destroy", lib().kv_budget_destroy(budget))
+
+
+def kv_budget_used(budget) -> int:
+    r = ctypes.c_uint64(0)
+    _check("kv_budget_used", lib().kv_budget_used(budget, ctypes.byref(r)))
+    return int(r.value)
+
+
 def kv_pool_destroy(pool) -> None:
     _check("kv_pool_destroy", lib().kv_pool_destroy(pool))
+    _callbacks.pop(pool, None)
 
 
 def kv_alloc_blocks(pool, layout: int, n: int) -> np.ndarray:
@@ -263,7 +352,7 @@ def kv_pool_stats(pool) -> dict:
         "pages_total": s.pages_total, "pages_unassigned": s.pages_unassigned,
         "blocks_used": list(s.blocks_used), "blocks_cached": list(s.blocks_cached),
         "blocks_capacity": list(s.blocks_capacity), "bytes_used": s.bytes_used,
-        "bytes_total": s.bytes_total,
+        "bytes_total": s.bytes_total, "bytes_mapped": s.bytes_mapped,
     }
 
 

@@ -63,6 +63,79 @@ class DevicePool:
             pass
 
 
+class _RawDevice:
+    """A device byte range seen through __cuda_array_interface__ (no ownership)."""
+
+    def __init__(self, ptr: int, nbytes: int):
+        self.__cuda_array_interface__ = {"shape": (nbytes,), "typestr": "|u1", "data": (ptr, False),
+                                         "version": 3}
+
+
+class VmmPool:
+    """A VMM-backed elastic pool (kv_pool_create_vmm, CUDA backend): the
+    library reserves the virtual range and maps physical chunks as blocks are
+    allocated.  ``pages`` views the whole range (n_pages x page_bytes); only
+    rows of allocated blocks may be touched."""
+
+    def __init__(self, virtual_bytes: int, page_bytes: int, block_size: int, layouts, physical_limit: int = 0,
+                 budget=None, shuffle_seed: int = 0, chunk_bytes: int = 0, device: str = "cuda"):
+        self.device = torch.device(device)
+        dev_index = self.device.index if self.device.index is not None else torch.cuda.current_device()
+        self.err = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.handle = K.kv_pool_create_vmm(virtual_bytes, block_size, layouts, self.err, page_bytes=page_bytes,
+                                           shuffle_seed=shuffle_seed, chunk_bytes=chunk_bytes,
+                                           physical_limit=physical_limit, budget=budget, device=dev_index)
+        self.base = K.kv_pool_get_base(self.handle)
+        st = K.kv_pool_stats(self.handle)
+        self.page_bytes = int(page_bytes)
+        self.n_pages = int(st["pages_total"])
+        raw = torch.as_tensor(_RawDevice(self.base, self.n_pages * self.page_bytes), device=self.device)
+        self.pages = raw.view(self.n_pages, self.page_bytes)
+
+    def write_pages(self, ids, data_u16: np.ndarray) -> None:
+        """Rows of the given page ids (allocated blocks' first pages) <- data."""
+        idx = torch.as_tensor(np.asarray(ids, np.int64), device=self.device)
+        src = torch.from_numpy(np.ascontiguousarray(data_u16).view(np.uint8)).to(self.device)
+        self.pages.index_copy_(0, idx, src.view(len(idx), -1))
+
+    def fill_random(self, ids, seed: int) -> None:
+        """Finite bf16 values (N(0,1) rounded) in the given pages."""
+        g = torch.Generator(device=self.device)
+        g.manual_seed(seed)
+        idx = torch.as_tensor(np.asarray(ids, np.int64), device=self.device)
+        vals = torch.randn((len(idx), self.page_bytes // 2), generator=g, device=self.device).to(torch.bfloat16)
+        self.pages.index_copy_(0, idx, vals.view(torch.uint8))
+
+    def read_pages(self, ids) -> np.ndarray:
+        idx = torch.as_tensor(np.asarray(ids, np.int64), device=self.device)
+        return self.pages.index_select(0, idx).cpu().numpy().view(np.uint16)
+
+    def stats(self) -> dict:
+        return K.kv_pool_stats(self.handle)
+
+    def trim(self) -> int:
+        return K.kv_pool_trim(self.handle)
+
+    def error(self, stream=None) -> int:
+        return K.kv_pool_get_error(self.handle, stream)
+
+    def set_variant(self, v: int) -> None:
+        K.kv_set_attn_variant(self.handle, v)
+
+    def close(self) -> None:
+        if self.handle:
+            torch.cuda.synchronize()
+            self.pages = None
+            K.kv_pool_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 class DeviceBatch:
     """One layout's decode batch on the device (q, new K/V rows, table,
     lengths, output, workspace)."""
