@@ -52,6 +52,7 @@ namespace kvp {
 constexpr int kWarps = 8;  // each warp streams and computes its own units
 constexpr int kThreads = kWarps * 32;
 constexpr int kTile = 16;                         // tokens per unit
+constexpr int kMinUnitsPerPart = 4;
 constexpr uint32_t kHalfBytes = kTile * 128;      // one 64-column box: 16 rows x 128 B
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
@@ -648,9 +649,12 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // The W units are cut into NP = min(P * kWarps, W) equal parts; part i is
     // [i*W/NP, (i+1)*W/NP) and belongs to warp i % kWarps of CTA i / kWarps.
     // With NP <= W every part is non-empty, so a run's contributors are
-    // exactly the parts part_of(first unit) .. part_of(last unit).
+    // exactly the parts part_of(first unit) .. part_of(last unit).  A part
+    // gets at least kMinUnitsPerPart units when the batch is small (fewer
+    // partials to write and merge; enough warps still stream to fill HBM).
     const int64_t W = T[S];
-    const int64_t NP = W < (int64_t)a.P * kWarps ? W : (int64_t)a.P * kWarps;
+    const int64_t np_min = W > 0 ? (W / kMinUnitsPerPart > 0 ? W / kMinUnitsPerPart : 1) : 0;
+    const int64_t NP = np_min < (int64_t)a.P * kWarps ? np_min : (int64_t)a.P * kWarps;
     const int64_t first_part = (int64_t)blockIdx.x * kWarps;
     if (first_part >= NP) return;
     const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
@@ -771,21 +775,31 @@ struct CombineArgs {
     int32_t KS;
 };
 
+constexpr int kCombineMaxThreads = 1024;
+
+// Thread groups per combine CTA: at least enough for 256 threads, more when
+// runs are expected to carry many records (about 8 records per thread), up
+// to 1024 threads.
 template <int D, int G>
-__host__ __device__ constexpr int combine_groups() { return (G * D / 4) >= 256 ? 1 : 256 / (G * D / 4); }
-template <int D, int G>
-__host__ __device__ constexpr int combine_threads() { return (G * D / 4) * combine_groups<D, G>(); }
+inline int combine_groups(double records_per_run)
+{
+    constexpr int NC = G * D / 4;
+    const int base = NC >= 256 ? 1 : 256 / NC;
+    const int most = kCombineMaxThreads / NC;
+    int want = (int)(records_per_run / 8.0 + 0.999);
+    return want < base ? base : (want > most ? most : want);
+}
 
 template <int D, int G>
-__global__ void __launch_bounds__(combine_threads<D, G>()) combine_kernel(const __grid_constant__ CombineArgs c)
+__global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __grid_constant__ CombineArgs c)
 {
     constexpr uint32_t MF = merge_floats<D, G>();
     constexpr int NC = G * D / 4;  // float4 columns of a run's output
-    constexpr int NG = combine_groups<D, G>();
-    constexpr int T = NC * NG;
-    __shared__ float s_M[NG > 1 ? T : 1];
-    __shared__ float s_L[NG > 1 ? T : 1];
-    __shared__ float4 s_O[NG > 1 ? T : 1];
+    static_assert(NC <= kCombineMaxThreads, "one thread per output column");
+    const int NG = (int)blockDim.x / NC;  // groups of NC threads
+    __shared__ float s_M[kCombineMaxThreads];
+    __shared__ float s_L[kCombineMaxThreads];
+    __shared__ float4 s_O[kCombineMaxThreads];
     const int r = blockIdx.x;
     grid_dependency_wait();  // the attention grid's partials and run table
     const int2 info = c.ws_run[r];
@@ -818,7 +832,7 @@ __global__ void __launch_bounds__(combine_threads<D, G>()) combine_kernel(const 
         O.w = O.w * sa + ok.w * sb;
         M = Mn;
     }
-    if constexpr (NG > 1) {
+    if (NG > 1) {
         s_M[tid] = M;
         s_L[tid] = L;
         s_O[tid] = O;
