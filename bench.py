@@ -59,11 +59,13 @@ class ClockSampler:
         self.lines = []
         self.thread = None
 
-    def start(self):
+    def start(self, cores=None):
+        """cores: CPU set for the nvidia-smi child (default: this thread's)"""
+        pre = (lambda: os.sched_setaffinity(0, cores)) if cores else None
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True, preexec_fn=pre)
         except Exception:
             self.proc = None
             return
@@ -102,6 +104,28 @@ class ClockSampler:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+
+def pin_process(local_rank: int):
+    """Keep this process on four cores (a set per local rank), set before
+    torch and the CUDA driver start their threads so that every thread
+    created later inherits it.  With the submitting thread and the driver's
+    threads free to spread over the cores, the step's launches reached the
+    GPU late enough to cost the programmatic overlap of consecutive kernels
+    (measured on a GB300 machine, config 2: 37 us of host time and 63 us per
+    step unpinned, 23 us and 58.5 us pinned).  Returns the cores, or None."""
+    try:
+        allowed = sorted(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return None
+    if len(allowed) < 8:
+        return None
+    cores = {allowed[(2 + 4 * local_rank + i) % len(allowed)] for i in range(4)}
+    try:
+        os.sched_setaffinity(0, cores)
+    except OSError:
+        return None
+    return sorted(cores)
 
 
 def aggregate_ranks(dist, device, ms: float, e2e_ms: float, units: dict) -> tuple:
@@ -380,6 +404,11 @@ def main():
         run_reference(args, rank, world)
         return
 
+    try:
+        all_cores = os.sched_getaffinity(0)
+    except (AttributeError, OSError):
+        all_cores = None
+    pinned_cores = pin_process(local)  # before torch / CUDA create their threads
     import torch
 
     torch.cuda.set_device(local)
@@ -429,25 +458,31 @@ def main():
         launches_per_step = n
         return nbytes
 
+    # the clock sampler starts first; the warm-up steps then run right before
+    # the timed region, so the GPU enters it busy rather than after an idle gap
+    clocks = ClockSampler(local)
+    clocks.start(cores=all_cores if pinned_cores else None)  # the sampler stays off the pinned cores' load
+    time.sleep(0.3)
     for i in range(args.warmup):
         step()
-    torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    clocks = ClockSampler(local)
-    clocks.start()
-    time.sleep(0.3)
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # the attention call is timed with an event pair on every SAMPLE-th step
+    # only: an event between two kernels ends their programmatic overlap, so
+    # pairs on every step would slow the step they are meant to measure
+    SAMPLE = 10
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range((args.steps + SAMPLE - 1) // SAMPLE)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     step_bytes = []
+    h0 = time.perf_counter()
     t_start.record(stream)
     for i in range(args.steps):
-        step_bytes.append(step(evs[i]))
+        step_bytes.append(step(evs[i // SAMPLE] if i % SAMPLE == 0 else None))
     t_end.record(stream)
+    host_us = (time.perf_counter() - h0) * 1e6 / args.steps  # host submission time per step
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
@@ -457,7 +492,8 @@ def main():
     dram_rank = sum(x[0] for x in step_bytes)
     logical_rank = sum(x[1] for x in step_bytes)
     attn_avg_ms = float(np.mean(attn_ms))
-    attn_gbs = dram_rank / args.steps / (attn_avg_ms * 1e-3) / 1e9  # this rank's kernels
+    sampled = [step_bytes[i][0] for i in range(0, args.steps, SAMPLE)]
+    attn_gbs = float(np.mean(sampled)) / (attn_avg_ms * 1e-3) / 1e9  # this rank's kernels
     peak, peak_kind = load_peaks()
 
     # end to end: q / k / v from pinned host memory, output back to host, every step
@@ -530,10 +566,14 @@ def main():
         "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peak, "unit": "GB/s",
                      "frac": attn_gbs / peak, "traffic": traffic,
                      "kernel": "paged_attn_kernel (+ combine_kernel, fused append)",
-                     "peak_kind": peak_kind, "attn_ms": attn_avg_ms},
+                     "peak_kind": peak_kind, "attn_ms": attn_avg_ms,
+                     "timed_launches": len(attn_ms), "timing": f"CUDA events around every {SAMPLE}th step's "
+                                                                 "attention call in the timed region"},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,
+        "host_us_per_step": host_us,
+        "host_cores": pinned_cores,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,

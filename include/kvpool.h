@@ -308,7 +308,9 @@ int kv_seq_trim(kv_seqtab *t, int s);
  * since the previous sync (of this table, to any device copy) goes to
  * dev_table (int32 [max_seqs][max_blocks]).  The values travel as kernel
  * parameters, so the host table may change right after the call returns.
- * The first sync after create sends the whole table.
+ * The first sync after create sends the whole table.  The sync kernel is a
+ * programmatic dependent of the previous work in the stream: its launch
+ * overlaps that work, and it waits for it to complete before writing.
  */
 int kv_seqtab_sync(kv_seqtab *t, int32_t *dev_table, int32_t *dev_ctx_lens, void *stream);
 

@@ -776,10 +776,13 @@ struct CombineArgs {
 };
 
 constexpr int kCombineMaxThreads = 1024;
+constexpr int kCombineBatch = 8;  // records each thread loads per round trip
 
-// Thread groups per combine CTA: at least enough for 256 threads, more when
-// runs are expected to carry many records (about 8 records per thread), up
-// to 1024 threads.
+// Thread groups per combine CTA: at least enough for 256 threads (a run's
+// records are spread over the groups, kCombineBatch loads in flight per
+// thread; at 64 registers four such CTAs fit on an SM, so one wave covers
+// 600 runs), more when runs are expected to carry many records (about 8
+// records per thread), up to 1024 threads.
 template <int D, int G>
 inline int combine_groups(double records_per_run)
 {
@@ -801,6 +804,9 @@ __global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __gri
     __shared__ float s_L[kCombineMaxThreads];
     __shared__ float4 s_O[kCombineMaxThreads];
     const int r = blockIdx.x;
+    // the next grid in the stream may be scheduled now; it waits for this
+    // one to complete before touching anything this grid reads
+    grid_launch_dependents();
     grid_dependency_wait();  // the attention grid's partials and run table
     const int2 info = c.ws_run[r];
     const int s = r / c.Hkv, g = r % c.Hkv;
@@ -813,24 +819,37 @@ __global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __gri
     const int col = tid % NC;
     const int grp = tid / NC;
     const int h = (col * 4) / D;
-    // online merge of this group's records: M running max, L and O relative to M
+    // online merge of this group's records: M running max, L and O relative
+    // to M; records k = grp, grp + NG, ... are loaded kCombineBatch at a time
     float M = -INFINITY, L = 0.f;
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-    for (int k = grp; k < cnt; k += NG) {
-        const float *sl = k < npre ? c.ws_pre + (((int64_t)k * c.S + s) * c.Hkv + g) * MF
-                                   : base + (int64_t)(k - npre) * MF;
-        const float mk = sl[G * D + h];
-        const float lk = sl[G * D + G + h];
-        const float4 ok = *reinterpret_cast<const float4 *>(sl + col * 4);
-        const float Mn = fmaxf(M, mk);
-        const float sa = fast_exp2(M - Mn), sb = fast_exp2(mk - Mn);
-        L = L * sa + lk * sb;
-        O.x = O.x * sa + ok.x * sb;
-        O.y = O.y * sa + ok.y * sb;
-        O.z = O.z * sa + ok.z * sb;
-        O.w = O.w * sa + ok.w * sb;
-        M = Mn;
+    for (int k0 = grp; k0 < cnt; k0 += NG * kCombineBatch) {
+        float mv[kCombineBatch], lv[kCombineBatch];
+        float4 ov[kCombineBatch];
+#pragma unroll
+        for (int b = 0; b < kCombineBatch; ++b) {
+            const int k = k0 + b * NG;
+            mv[b] = -INFINITY;
+            if (k < cnt) {
+                const float *sl = k < npre ? c.ws_pre + (((int64_t)k * c.S + s) * c.Hkv + g) * MF
+                                           : base + (int64_t)(k - npre) * MF;
+                mv[b] = sl[G * D + h];
+                lv[b] = sl[G * D + G + h];
+                ov[b] = *reinterpret_cast<const float4 *>(sl + col * 4);
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < kCombineBatch; ++b) {
+            if (mv[b] == -INFINITY) continue;  // past the run's records
+            const float Mn = fmaxf(M, mv[b]);
+            const float sa = fast_exp2(M - Mn), sb = fast_exp2(mv[b] - Mn);
+            L = L * sa + lv[b] * sb;
+            O.x = O.x * sa + ov[b].x * sb;
+            O.y = O.y * sa + ov[b].y * sb;
+            O.z = O.z * sa + ov[b].z * sb;
+            O.w = O.w * sa + ov[b].w * sb;
+            M = Mn;
+        }
     }
     if (NG > 1) {
         s_M[tid] = M;

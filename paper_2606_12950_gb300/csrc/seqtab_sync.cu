@@ -27,6 +27,10 @@ __global__ void seqtab_sync_kernel(const __grid_constant__ SyncParams<WORDS> p)
     // a following programmatic-dependent grid may launch now; it waits for
     // this grid to complete before it reads the table or the lengths
     asm volatile("griddepcontrol.launch_dependents;" :::);
+    // this grid is itself launched as a programmatic dependent (its launch
+    // overlaps the previous kernel): wait for that kernel, which may still
+    // read the lengths and the table, before writing them
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int i = threadIdx.x; i < p.n_lens; i += blockDim.x) p.dev_lens[p.lens_begin + i] = p.data[i];
     for (int j = threadIdx.x; j < p.n_patches; j += blockDim.x)
         p.dev_table[p.data[p.n_lens + 2 * j]] = p.data[p.n_lens + 2 * j + 1];
@@ -50,8 +54,16 @@ int launch_chunk(kv_seqtab *t, int32_t *dev_table, int32_t *dev_lens, size_t li,
         p.data[nl + 2 * j] = idx;
         p.data[nl + 2 * j + 1] = t->table[(size_t)idx];
     }
-    seqtab_sync_kernel<WORDS><<<1, 256, 0, st>>>(p);
-    return cudaGetLastError() == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, seqtab_sync_kernel<WORDS>, p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
 constexpr int kSmallWords = 256;
