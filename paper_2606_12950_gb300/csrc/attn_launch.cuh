@@ -14,6 +14,26 @@ namespace kvp {
 // CTA's units resolved in the prologue) is kRowsCap entries
 constexpr size_t kSmemMax = 227 * 1024;
 
+// Resident CTAs per SM of kernel fn at this block size and dynamic shared
+// memory, queried once per (instantiation, shared-memory size) and cached:
+// the runtime query costs microseconds of host time on every launch.
+template <class Fn>
+int cached_occupancy(Fn fn, int threads, size_t smem, int *occ)
+{
+    static std::atomic<long long> key{-1};
+    static std::atomic<int> val{0};
+    if (key.load(std::memory_order_acquire) == (long long)smem) {
+        *occ = val.load(std::memory_order_relaxed);
+        return KV_OK;
+    }
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, threads, smem) != cudaSuccess) return KV_ERR_CUDA;
+    val.store(o, std::memory_order_relaxed);
+    key.store((long long)smem, std::memory_order_release);
+    *occ = o;
+    return KV_OK;
+}
+
 template <int D, int G, class Comp>
 int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaStream_t st, bool launch,
              int *P_out)
@@ -28,7 +48,7 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     const size_t smem = attn_smem_bytes<D, G>(a.S, kRowsCap);
     if (smem > kSmemMax) return KV_ERR_INVALID_ARG;  // S too large for the per-CTA sequence index
     int occ = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, kThreads, smem) != cudaSuccess) return KV_ERR_CUDA;
+    if (cached_occupancy(fn, kThreads, smem, &occ) != KV_OK) return KV_ERR_CUDA;
     const int P = P_req > 0 ? P_req : std::max(1, occ) * std::max(1, sm_count);
     *P_out = P;
     if (!launch) return KV_OK;
@@ -76,8 +96,7 @@ int cascade_run(const CUtensorMap *tmap, const CascadeArgs *c, int grid, int sm_
     }
     if (!launch) {
         int occ = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, kPreThreads, smem) != cudaSuccess)
-            return KV_ERR_CUDA;
+        if (cached_occupancy(fn, kPreThreads, smem, &occ) != KV_OK) return KV_ERR_CUDA;
         *P_out = std::max(1, occ) * std::max(1, sm_count);
         return KV_OK;
     }

@@ -7,9 +7,14 @@
 // contraction per KV head: all sharers' query heads of that KV head form the
 // rows, the prefix tokens the columns.  The prefix K/V is then read once per
 // (row tile, key split) from L2 instead of once per sharer, and the work runs
-// on the tensor cores as a small flash-attention forward:
-//   S = Q K^T (m16n8k16 bf16 -> fp32), online softmax in base 2,
-//   O += P V, per 64-key tile streamed through a 3-stage TMA pipeline.
+// on the fifth-generation tensor cores as a small flash-attention forward:
+//   S = Q K^T     tcgen05.mma, M = 128 query rows, N = 64 keys, fp32 in TMEM
+//   softmax       one thread per row, S read from TMEM, base 2, lazy rescale
+//   O += P V      tcgen05.mma, P (bf16) from shared memory, O in TMEM
+// with 64-key K/V tiles streamed by TMA through a 3-stage ring.  A CTA holds
+// two Q tiles that share every K/V tile: while one tile's four warps run
+// the softmax, the tensor core works on the other tile.  One thread issues
+// the TMA loads, one thread issues the MMAs, one thread owns each row.
 // Each CTA leaves, per (sharer, KV head), one fp32 record (unnormalised o,
 // running max m, sum l) in the same format as the decode kernel's split
 // partials; the combine kernel merges prefix and suffix records, which is
@@ -21,14 +26,16 @@
 
 namespace kvp {
 
-constexpr int kPreWarps = 4;
-constexpr int kPreThreads = kPreWarps * 32;
-constexpr int kPreRows = kPreWarps * 16;  // query rows (sharer, head) per CTA
-constexpr int kPreKeys = 64;              // prefix tokens per pipeline tile
+constexpr int kPreRows = 128;             // query rows (sharer, head) per Q tile: the MMA's M
+constexpr int kPreQTiles = 2;             // Q tiles per CTA, sharing every K/V tile
+constexpr int kPreKeys = 64;              // prefix tokens per pipeline tile: S's N, P.V's K
 constexpr int kPreStages = 3;
-constexpr int kPreRowsCap = 1024;         // 16-token sub-tiles resolved up front
+constexpr int kPreSoftWarps = 4;          // per Q tile: one thread per query row
+constexpr int kPreThreads = (kPreQTiles * kPreSoftWarps + 2) * 32;  // + TMA warp + MMA warp
+constexpr int kPreRowsCap = 256;          // 16-token sub-tiles resolved up front
 constexpr int kMaxKeySplits = 8;
 constexpr int kCascadeWords = 4080;       // plan words carried as kernel parameters
+constexpr uint32_t kPreTmemCols = 256;    // per Q tile: S0 [0,64), S1 [64,128), O [128, 128 + d)
 
 struct CascadeArgs {
     const uint16_t *q;
@@ -53,9 +60,10 @@ struct CascadeArgs {
     int32_t data[kCascadeWords];
 };
 
-// rows per row tile: whole query-head groups of consecutive members
+// members per CTA: whole query-head groups of consecutive members in each of
+// its Q tiles
 template <int G>
-__host__ __device__ constexpr int pre_members_per_tile() { return kPreRows / G; }
+__host__ __device__ constexpr int pre_members_per_tile() { return kPreQTiles * (kPreRows / G); }
 
 // Pool row (TMA y) of the K sub-tile holding prefix tokens 16q .. 16q+15 for
 // KV head g, read from the lead member's table; -1 if outside the pool.
@@ -73,26 +81,59 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// shared-memory layout of the prefix kernel (offsets from a 1024-byte aligned
+// base): Q [tiles][halves][128 rows][128 B] | P [tiles][128 rows][128 B] |
+// stages x (K, V) [halves][64 keys][128 B] | mbarriers | TMEM address |
+// sub-tile rows
+template <int D>
+struct PreSmem {
+    static constexpr int HALVES = D / 64;
+    static constexpr uint32_t KV_HALF = kPreKeys * 128;       // 64 keys x 64 columns
+    static constexpr uint32_t KV_TILE = HALVES * KV_HALF;     // K (or V) of one key tile
+    static constexpr uint32_t STAGE = 2 * KV_TILE;
+    static constexpr uint32_t Q_HALF = kPreRows * 128;
+    static constexpr uint32_t Q_TILE = HALVES * Q_HALF;
+    static constexpr uint32_t P_TILE = kPreRows * 128;        // 128 rows x 64 keys bf16
+    static constexpr uint32_t Q_OFF = 0;
+    static constexpr uint32_t P_OFF = kPreQTiles * Q_TILE;
+    static constexpr uint32_t ST_OFF = P_OFF + kPreQTiles * P_TILE;
+    static constexpr uint32_t BAR_OFF = ST_OFF + kPreStages * STAGE;
+    // full, empty per stage; per Q tile: s_full x2, s_free x2, p_full, o_done; fin; q_ready
+    static constexpr int NBARS = 2 * kPreStages + 6 * kPreQTiles + 2;
+    static constexpr uint32_t SLOT_OFF = BAR_OFF + NBARS * 8;
+    static constexpr uint32_t ROWS_OFF = SLOT_OFF + 16;
+    static constexpr uint32_t BYTES = ROWS_OFF + kPreRowsCap * 4;
+};
+
 template <int D, int G>
-__global__ void __launch_bounds__(kPreThreads)
+__global__ void __launch_bounds__(kPreThreads, 1)
 cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CascadeArgs c)
 {
-    constexpr int HALVES = D / 64;
-    constexpr uint32_t SUB_BYTES = HALVES * kHalfBytes;           // 16 tokens x D
-    constexpr uint32_t KT_BYTES = (kPreKeys / kTile) * SUB_BYTES;  // 64 tokens x D
-    constexpr uint32_t STAGE_BYTES = 2 * KT_BYTES;                 // K then V
+    using L = PreSmem<D>;
+    constexpr int HALVES = L::HALVES;
     constexpr uint32_t MF = merge_floats<D, G>();
-    constexpr int MT = pre_members_per_tile<G>();
-    constexpr int KSL = D / 16;        // k-slices of q.K
-    constexpr int NT = kPreKeys / 8;   // key n-tiles of S
-    constexpr int ND = D / 8;          // d n-tiles of O
+    constexpr int MQ = kPreRows / G;         // members per Q tile
+    constexpr int MT = pre_members_per_tile<G>();  // members per CTA (kPreQTiles Q tiles)
+    constexpr int NSUB = kPreKeys / kTile;   // 16-token sub-tiles per key tile
+    constexpr uint32_t O_COL = 2 * kPreKeys;  // within a Q tile's TMEM columns
+    constexpr int SOFT_THREADS = kPreQTiles * kPreSoftWarps * 32;
+    static_assert(O_COL + D <= kPreTmemCols, "S double buffer and O fit a Q tile's TMEM columns");
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kPreStages * STAGE_BYTES);
-    int32_t *rows = reinterpret_cast<int32_t *>(bars + kPreStages);  // [kPreRowsCap]
+    const uint32_t sbase = smem_u32(smem);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L::BAR_OFF);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + L::SLOT_OFF);
+    int32_t *rows = reinterpret_cast<int32_t *>(smem + L::ROWS_OFF);
+    auto bar = [&](int i) { return smem_u32(&bars[i]); };
+    constexpr int FULL = 0, EMPTY = kPreStages, QB = 2 * kPreStages, FIN = QB + 6 * kPreQTiles, Q_READY = FIN + 1;
+    // per Q tile a: S_FULL(a, b) = QB + 6a + b, S_FREE(a, b) = QB + 6a + 2 + b, P_FULL(a) = QB + 6a + 4,
+    // O_DONE(a) = QB + 6a + 5
+    auto s_full = [&](int a, int b) { return bar(QB + 6 * a + b); };
+    auto s_free = [&](int a, int b) { return bar(QB + 6 * a + 2 + b); };
+    auto p_full = [&](int a) { return bar(QB + 6 * a + 4); };
+    auto o_done = [&](int a) { return bar(QB + 6 * a + 5); };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int gid = lane >> 2, tig = lane & 3;
     int bid = blockIdx.x;
     const int ks = bid % c.KS;
     bid /= c.KS;
@@ -106,196 +147,270 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     const int32_t *skip = members + c.n_members;
     int grp = 0;
     while (grp + 1 < c.n_groups && tile_off[grp + 1] <= tile) ++grp;
-    const int m0 = mem_off[grp] + (tile - tile_off[grp]) * MT;  // this tile's members [m0, m1)
+    const int m0 = mem_off[grp] + (tile - tile_off[grp]) * MT;  // this CTA's members [m0, m1)
     const int m1 = min(m0 + MT, mem_off[grp + 1]);
     const int lead = members[mem_off[grp]];
     const int kt_all = tokens[grp] / kPreKeys;
     const int kt0 = ks * kt_all / c.KS, kt1 = (ks + 1) * kt_all / c.KS;  // non-empty: KS <= kt_all
     const int nkt = kt1 - kt0;
+    const int nsub = nkt * NSUB;
 
     if (tid == 0) {
-        for (int i = 0; i < kPreStages; ++i) mbar_init(smem_u32(&bars[i]), 1);
+        for (int i = 0; i < kPreStages; ++i) {
+            mbar_init(bar(FULL + i), 1);
+            mbar_init(bar(EMPTY + i), 1);
+        }
+        for (int a = 0; a < kPreQTiles; ++a) {
+            for (int b = 0; b < 2; ++b) {
+                mbar_init(s_full(a, b), 1);
+                mbar_init(s_free(a, b), kPreSoftWarps * 32);
+            }
+            mbar_init(p_full(a), kPreSoftWarps * 32);
+            mbar_init(o_done(a), 1);
+        }
+        mbar_init(bar(FIN), 1);
+        mbar_init(bar(Q_READY), SOFT_THREADS);
         fence_mbar_init();
     }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(tslot), kPreQTiles * kPreTmemCols);
+        tmem_relinquish();
+    }
     if (tid == 32) prefetch_tensormap(&tmap);
+    // barriers initialised and TMEM allocated: everything below may use them
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tslot;
+    bool dead = false;
+    constexpr int TMA_WARP = kPreQTiles * kPreSoftWarps, MMA_WARP = TMA_WARP + 1;
     grid_launch_dependents();
     grid_dependency_wait();  // the table (and q) come from the grids before
 
     if (blockIdx.x == 0)
         for (int s = tid; s < c.S; s += kPreThreads) c.ws_skip[s] = skip[s];
-    const int nsub = nkt * (kPreKeys / kTile);
-    for (int i = tid; i < min(nsub, kPreRowsCap); i += kPreThreads)
-        rows[i] = pre_sub_row(c, lead, g, kt0 * (kPreKeys / kTile) + i);
-    __syncthreads();
 
-    // K and V of key tile i (relative to kt0) into stage st; thread 0 only
-    auto issue = [&](int st, int i) {
-        const uint32_t kdst = smem_u32(smem + st * STAGE_BYTES), vdst = kdst + KT_BYTES;
-        const uint32_t bar = smem_u32(&bars[st]);
-        int32_t y[kPreKeys / kTile];
-        bool ok = true;
-#pragma unroll
-        for (int j = 0; j < kPreKeys / kTile; ++j) {
-            const int32_t q = i * (kPreKeys / kTile) + j;
-            y[j] = q < kPreRowsCap ? rows[q] : pre_sub_row(c, lead, g, kt0 * (kPreKeys / kTile) + q);
-            ok = ok && y[j] >= 0;
-        }
-        if (!ok) {
-            report(c.err, KV_ERR_DEVICE_BOUNDS);
-            mbar_arrive(bar);  // complete the phase without data
-            return;
-        }
-        const uint64_t pol = l2_policy_evict_normal();  // the prefix is re-read by every row tile
-        mbar_arrive_expect_tx(bar, STAGE_BYTES);
-#pragma unroll
-        for (int j = 0; j < kPreKeys / kTile; ++j)
-#pragma unroll
-            for (int h = 0; h < HALVES; ++h) {
-                const uint32_t off = j * SUB_BYTES + h * kHalfBytes;
-                tma_load_2d(kdst + off, &tmap, h * 64, y[j], bar, pol);
-                tma_load_2d(vdst + off, &tmap, h * 64, y[j] + c.Hkv * c.bs, bar, pol);
-            }
-    };
-    if (tid == 0)
-        for (int i = 0; i < kPreStages && i < nkt; ++i) issue(i, i);
-
-    // Q fragments (A operand, row-major 16 x 16 per k-slice) straight from global
-    const int r0 = warp * 16 + gid, r1 = r0 + 8;
-    const int mi0 = m0 + r0 / G, mi1 = m0 + r1 / G;
-    const bool v0 = r0 < MT * G && mi0 < m1, v1 = r1 < MT * G && mi1 < m1;
+    // Q rows (member, head) of KV head g into the swizzled K-major layout the
+    // MMA reads: softmax thread t fills row t % 128 of Q tile t / 128; rows
+    // past the CTA's members are zero.  The MMA thread waits for q_ready.
     const int Hq = c.Hkv * G;
-    const uint16_t *q0 = v0 ? c.q + ((int64_t)members[mi0] * Hq + (int64_t)g * G + r0 % G) * D : nullptr;
-    const uint16_t *q1 = v1 ? c.q + ((int64_t)members[mi1] * Hq + (int64_t)g * G + r1 % G) * D : nullptr;
-    uint32_t qa[KSL][4];
+    const int qa_tile = tid / kPreRows, r = tid % kPreRows;  // Q tile and row of a softmax thread
+    const int mrow = m0 + qa_tile * MQ + r / G;               // its member index
+    const bool row_ok = tid < SOFT_THREADS && r < MQ * G && mrow < m1;
+    if (tid < SOFT_THREADS) {
+        const uint16_t *qrow = row_ok ? c.q + ((int64_t)members[mrow] * Hq + (int64_t)g * G + r % G) * D : nullptr;
+        uint8_t *qdst = smem + L::Q_OFF + qa_tile * L::Q_TILE;
+        uint4 qv[D / 8];
 #pragma unroll
-    for (int kk = 0; kk < KSL; ++kk) {
-        const int col = kk * 16 + 2 * tig;
-        qa[kk][0] = v0 ? *reinterpret_cast<const uint32_t *>(q0 + col) : 0u;
-        qa[kk][1] = v1 ? *reinterpret_cast<const uint32_t *>(q1 + col) : 0u;
-        qa[kk][2] = v0 ? *reinterpret_cast<const uint32_t *>(q0 + col + 8) : 0u;
-        qa[kk][3] = v1 ? *reinterpret_cast<const uint32_t *>(q1 + col + 8) : 0u;
+        for (int ch = 0; ch < D / 8; ++ch)
+            qv[ch] = row_ok ? *reinterpret_cast<const uint4 *>(qrow + ch * 8) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int ch = 0; ch < D / 8; ++ch)
+            *reinterpret_cast<uint4 *>(qdst + (ch / 8) * L::Q_HALF + swz(r, ch % 8)) = qv[ch];
+        fence_proxy_async_smem();  // Q (generic stores) is read by the tensor cores
+        mbar_arrive(bar(Q_READY));
     }
 
-    float o[ND][4];
-#pragma unroll
-    for (int nd = 0; nd < ND; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
-    float mr0 = -INFINITY, mr1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    bool dead = false;
-
-    for (int i = 0; i < nkt; ++i) {
-        const int st = i % kPreStages;
-        wait_phase(smem_u32(&bars[st]), (uint32_t)(i / kPreStages) & 1u, c.err, dead);
-        const uint32_t kb = smem_u32(smem + st * STAGE_BYTES), vb = kb + KT_BYTES;
-        if (!dead) {
-            // ---- S = Q K^T over 64 keys ----
-            float s[NT][4];
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-#pragma unroll
-            for (int kk = 0; kk < KSL; ++kk)
-#pragma unroll
-                for (int nt = 0; nt < NT; nt += 2) {
-                    const int key = (nt + (lane >> 4)) * 8 + (lane & 7);
-                    const int chunk = 2 * kk + ((lane >> 3) & 1);
-                    uint32_t b0, b1, b2, b3;
-                    ldmatrix_x4(kb + (key >> 4) * SUB_BYTES + swz(key & 15, chunk), b0, b1, b2, b3);
-                    mma_bf16_16816(s[nt], qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], b0, b1);
-                    mma_bf16_16816(s[nt + 1], qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], b2, b3);
+    if (warp == TMA_WARP) {
+        // ---- TMA producer warp: resolves the pool rows of the CTA's key range
+        // from the block table, then streams K and V of key tile t into stage
+        // t % stages, each lane issuing some of the stage's boxes (one
+        // issuing thread per SM cannot keep the loads flowing) ----
+        for (int i = lane; i < min(nsub, kPreRowsCap); i += 32) rows[i] = pre_sub_row(c, lead, g, kt0 * NSUB + i);
+        __syncwarp();
+        const uint64_t pol = l2_policy_evict_normal();  // the prefix is re-read by every row tile
+        constexpr int NBOX = NSUB * HALVES;               // boxes of K (and of V) per key tile
+        for (int t = 0; t < nkt; ++t) {
+            const int st = t % kPreStages;
+            if (t >= kPreStages) wait_phase(bar(EMPTY + st), (uint32_t)(t / kPreStages - 1) & 1u, c.err, dead);
+            const uint32_t kdst = sbase + L::ST_OFF + st * L::STAGE, vdst = kdst + L::KV_TILE;
+            int32_t y = 0;
+            bool ok = true;
+            if (lane < NBOX) {
+                const int32_t q = t * NSUB + lane / HALVES;
+                y = q < kPreRowsCap ? rows[q] : pre_sub_row(c, lead, g, kt0 * NSUB + q);
+                ok = y >= 0;
+            }
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) {
+                if (lane == 0) {
+                    report(c.err, KV_ERR_DEVICE_BOUNDS);
+                    mbar_arrive(bar(FULL + st));  // complete the phase without data
                 }
-            // ---- online softmax (base 2): rows r0 (c0, c1) and r1 (c2, c3) ----
-            float t0 = -INFINITY, t1 = -INFINITY;
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                s[nt][0] *= c.qk_scale;
-                s[nt][1] *= c.qk_scale;
-                s[nt][2] *= c.qk_scale;
-                s[nt][3] *= c.qk_scale;
-                t0 = fmaxf(t0, fmaxf(s[nt][0], s[nt][1]));
-                t1 = fmaxf(t1, fmaxf(s[nt][2], s[nt][3]));
+                __syncwarp();
+                continue;
             }
-#pragma unroll
-            for (int off = 1; off < 4; off <<= 1) {
-                t0 = fmaxf(t0, __shfl_xor_sync(0xffffffffu, t0, off));
-                t1 = fmaxf(t1, __shfl_xor_sync(0xffffffffu, t1, off));
+            if (lane == 0) mbar_arrive_expect_tx(bar(FULL + st), L::STAGE);
+            __syncwarp();
+            if (lane < NBOX) {
+                const int j = lane / HALVES, h = lane % HALVES;
+                const uint32_t off = h * L::KV_HALF + j * (kTile * 128);
+                tma_load_2d(kdst + off, &tmap, h * 64, y, bar(FULL + st), pol);
+                tma_load_2d(vdst + off, &tmap, h * 64, y + c.Hkv * c.bs, bar(FULL + st), pol);
             }
-            const float mn0 = fmaxf(mr0, t0), mn1 = fmaxf(mr1, t1);
-            const float a0 = fast_exp2(mr0 - mn0), a1 = fast_exp2(mr1 - mn1);
-            mr0 = mn0;
-            mr1 = mn1;
-            l0 *= a0;
-            l1 *= a1;
+            __syncwarp();
+        }
+        // drain: the last stages' loads have landed (already waited on by the
+        // MMA thread unless a wait ran out)
+        if (lane == 0)
+            for (int t = max(0, nkt - kPreStages); t < nkt; ++t)
+                wait_phase(bar(FULL + t % kPreStages), (uint32_t)(t / kPreStages) & 1u, c.err, dead);
+    } else if (warp == MMA_WARP && lane == 0) {
+        // ---- MMA issuer: per key tile j, S_{a,j} = Q_a K_j^T for both Q
+        // tiles, then O_a += P_{a,j-1} V_{j-1}; the tensor core works on one
+        // tile while the other tile's warps run the softmax ----
+        constexpr uint32_t ID_S = idesc_bf16_f32(kPreRows, kPreKeys, 0, 0);
+        constexpr uint32_t ID_O = idesc_bf16_f32(kPreRows, D, 0, 1);
+        wait_phase(bar(Q_READY), 0u, c.err, dead);
+        for (int j = 0; j <= nkt; ++j) {
+            if (j < nkt) {
+                const int st = j % kPreStages;
+                wait_phase(bar(FULL + st), (uint32_t)(j / kPreStages) & 1u, c.err, dead);
+                const uint32_t ka = sbase + L::ST_OFF + st * L::STAGE;
 #pragma unroll
-            for (int nd = 0; nd < ND; ++nd) {
-                o[nd][0] *= a0;
-                o[nd][1] *= a0;
-                o[nd][2] *= a1;
-                o[nd][3] *= a1;
-            }
-            uint32_t pa[NT / 2][4];  // P as A operand, one 16-key slice per entry
+                for (int a = 0; a < kPreQTiles; ++a) {
+                    if (j >= 2) wait_phase(s_free(a, j & 1), (uint32_t)((j >> 1) - 1) & 1u, c.err, dead);
+                    tc_fence_after();
+                    const uint32_t qa = sbase + L::Q_OFF + a * L::Q_TILE;
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const float p0 = fast_exp2(s[nt][0] - mn0), p1 = fast_exp2(s[nt][1] - mn0);
-                const float p2 = fast_exp2(s[nt][2] - mn1), p3 = fast_exp2(s[nt][3] - mn1);
-                l0 += p0 + p1;
-                l1 += p2 + p3;
-                pa[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16(p0, p1);
-                pa[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16(p2, p3);
-            }
-            // ---- O += P V ----
-#pragma unroll
-            for (int j = 0; j < NT / 2; ++j)
-#pragma unroll
-                for (int nd = 0; nd < ND; nd += 2) {
-                    const int key = 16 * j + ((lane >> 3) & 1) * 8 + (lane & 7);
-                    const int chunk = nd + (lane >> 4);
-                    uint32_t b0, b1, b2, b3;
-                    ldmatrix_x4_trans(vb + (key >> 4) * SUB_BYTES + swz(key & 15, chunk), b0, b1, b2, b3);
-                    mma_bf16_16816(o[nd], pa[j][0], pa[j][1], pa[j][2], pa[j][3], b0, b1);
-                    mma_bf16_16816(o[nd + 1], pa[j][0], pa[j][1], pa[j][2], pa[j][3], b2, b3);
+                    for (int kk = 0; kk < D / 16; ++kk)
+                        umma_bf16(tbase + a * kPreTmemCols + (uint32_t)(j & 1) * kPreKeys,
+                                  smem_desc_sw128(qa + (kk / 4) * L::Q_HALF + (kk % 4) * 32, 16, 1024),
+                                  smem_desc_sw128(ka + (kk / 4) * L::KV_HALF + (kk % 4) * 32, 16, 1024), ID_S,
+                                  kk > 0);
+                    umma_commit(s_full(a, j & 1));
                 }
-        }
-        // every warp is done with this stage: refill it with tile i + stages
-        fence_proxy_async_smem();
-        __syncthreads();
-        if (tid == 0 && i + kPreStages < nkt) issue(st, i + kPreStages);
-    }
-
-    // ---- this CTA's record per (sharer, KV head) ----
+            }
+            if (j >= 1) {
+                const int jj = j - 1, st = jj % kPreStages;
+                const uint32_t va = sbase + L::ST_OFF + st * L::STAGE + L::KV_TILE;
 #pragma unroll
-    for (int off = 1; off < 4; off <<= 1) {
-        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-    }
-    if (dead) return;
-    if (v0) {
-        float *rec = c.ws_pre + (((int64_t)ks * c.S + members[mi0]) * c.Hkv + g) * MF;
-        const int hl = r0 % G;
+                for (int a = 0; a < kPreQTiles; ++a) {
+                    wait_phase(p_full(a), (uint32_t)jj & 1u, c.err, dead);
+                    tc_fence_after();
+                    const uint32_t pa = sbase + L::P_OFF + a * L::P_TILE;
 #pragma unroll
-        for (int nd = 0; nd < ND; ++nd)
-            *reinterpret_cast<float2 *>(rec + hl * D + nd * 8 + 2 * tig) = make_float2(o[nd][0], o[nd][1]);
-        if (tig == 0) {
-            rec[G * D + hl] = mr0;
-            rec[G * D + G + hl] = l0;
+                    for (int kk = 0; kk < kPreKeys / 16; ++kk)
+                        umma_bf16(tbase + a * kPreTmemCols + O_COL, smem_desc_sw128(pa + kk * 32, 16, 1024),
+                                  smem_desc_sw128(va + kk * (16 * 128), L::KV_HALF, 1024), ID_O, jj > 0 || kk > 0);
+                    umma_commit(o_done(a));
+                }
+                umma_commit(bar(EMPTY + st));
+            }
+        }
+        // every MMA of this thread has completed before TMEM is released
+        umma_commit(bar(FIN));
+        wait_phase(bar(FIN), 0u, c.err, dead);
+    } else if (tid < SOFT_THREADS) {
+        // ---- softmax: thread tid owns row r of Q tile qa_tile (TMEM lane r) ----
+        const int a = qa_tile;
+        const uint32_t trow = tbase + a * kPreTmemCols + ((uint32_t)((warp % 4) * 32) << 16);
+        uint8_t *prow = smem + L::P_OFF + a * L::P_TILE;
+        const float scale = c.qk_scale;
+        float m_run = -INFINITY, l_run = 0.f;
+        for (int j = 0; j < nkt; ++j) {
+            wait_phase(s_full(a, j & 1), (uint32_t)(j >> 1) & 1u, c.err, dead);
+            tc_fence_after();
+            float x[kPreKeys];
+            {
+                uint32_t v[32];
+#pragma unroll
+                for (int hf = 0; hf < kPreKeys / 32; ++hf) {
+                    tmem_ld32(trow + (uint32_t)(j & 1) * kPreKeys + hf * 32, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) x[hf * 32 + i] = __uint_as_float(v[i]);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(s_free(a, j & 1));
+            // tile max of the raw scores as a tree (scale > 0 commutes with max)
+            float t8[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                float t = x[i];
+#pragma unroll
+                for (int k = 8 + i; k < kPreKeys; k += 8) t = fmaxf(t, x[k]);
+                t8[i] = t;
+            }
+            const float t = fmaxf(fmaxf(fmaxf(t8[0], t8[1]), fmaxf(t8[2], t8[3])),
+                                  fmaxf(fmaxf(t8[4], t8[5]), fmaxf(t8[6], t8[7]))) * scale;
+            // lazy rescale: keep the running max unless the tile exceeds it by
+            // more than 2^8 (o and l share the stale max, so the ratio is exact)
+            const bool grow = t > m_run + 8.f;
+            const float m_new = grow ? t : m_run;
+            float rs[4] = {0.f, 0.f, 0.f, 0.f};
+            uint32_t pk[kPreKeys / 2];
+#pragma unroll
+            for (int i = 0; i < kPreKeys; i += 2) {
+                const float p0 = fast_exp2(fmaf(x[i], scale, -m_new));
+                const float p1 = fast_exp2(fmaf(x[i + 1], scale, -m_new));
+                rs[(i >> 1) & 3] += p0 + p1;
+                pk[i / 2] = pack_bf16(p0, p1);
+            }
+            // P_{a,j-1} and O_a: the MMAs of key tile j-1 have completed
+            if (j >= 1) {
+                wait_phase(o_done(a), (uint32_t)(j - 1) & 1u, c.err, dead);
+                tc_fence_after();
+            }
+            if (grow) {
+                const float al = fast_exp2(m_run - m_new);  // 0 on the first tile
+                l_run *= al;
+                if (j >= 1) {
+                    uint32_t v[32];
+#pragma unroll
+                    for (int cb = 0; cb < D / 32; ++cb) {
+                        tmem_ld32(trow + O_COL + cb * 32, v);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * al);
+                        tmem_st32(trow + O_COL + cb * 32, v);
+                    }
+                    tmem_wait_st();
+                }
+                m_run = m_new;
+            }
+            l_run += (rs[0] + rs[1]) + (rs[2] + rs[3]);
+#pragma unroll
+            for (int ch = 0; ch < kPreKeys / 8; ++ch)
+                *reinterpret_cast<uint4 *>(prow + swz(r, ch)) =
+                    make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
+            fence_proxy_async_smem();  // P (generic stores) is read by the tensor cores
+            tc_fence_before();
+            mbar_arrive(p_full(a));
+        }
+        // ---- this CTA's record per (sharer, KV head) ----
+        wait_phase(o_done(a), (uint32_t)(nkt - 1) & 1u, c.err, dead);
+        tc_fence_after();
+        float *rec = row_ok ? c.ws_pre + (((int64_t)ks * c.S + members[mrow]) * c.Hkv + g) * MF : nullptr;
+        const int hl = r % G;
+        uint32_t v[32];
+#pragma unroll
+        for (int cb = 0; cb < D / 32; ++cb) {
+            tmem_ld32(trow + O_COL + cb * 32, v);
+            tmem_wait_ld();
+            if (row_ok && !dead)
+#pragma unroll
+                for (int i = 0; i < 32; i += 4)
+                    *reinterpret_cast<float4 *>(rec + hl * D + cb * 32 + i) =
+                        make_float4(__uint_as_float(v[i]), __uint_as_float(v[i + 1]), __uint_as_float(v[i + 2]),
+                                    __uint_as_float(v[i + 3]));
+        }
+        if (row_ok && !dead) {
+            rec[G * D + hl] = m_run;
+            rec[G * D + G + hl] = l_run;
         }
     }
-    if (v1) {
-        float *rec = c.ws_pre + (((int64_t)ks * c.S + members[mi1]) * c.Hkv + g) * MF;
-        const int hl = r1 % G;
-#pragma unroll
-        for (int nd = 0; nd < ND; ++nd)
-            *reinterpret_cast<float2 *>(rec + hl * D + nd * 8 + 2 * tig) = make_float2(o[nd][2], o[nd][3]);
-        if (tig == 0) {
-            rec[G * D + hl] = mr1;
-            rec[G * D + G + hl] = l1;
-        }
-    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tbase, kPreQTiles * kPreTmemCols);
 }
 
 template <int D>
 inline size_t cascade_smem_bytes()
 {
-    return 1024 + (size_t)kPreStages * 2 * (kPreKeys / kTile) * (D / 64) * kHalfBytes + kPreStages * 8 +
-           (size_t)kPreRowsCap * 4;
+    return 1024 + (size_t)PreSmem<D>::BYTES;
 }
 
 }  // namespace kvp

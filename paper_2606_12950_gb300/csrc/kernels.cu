@@ -282,11 +282,14 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         nm += gr.count;
     }
     if (nm > S || 2 * (ng + 1) + ng + nm + S > kvp::kCascadeWords) return KV_ERR_INVALID_ARG;
-    auto c = std::make_unique<kvp::CascadeArgs>();
+    // the plan's parameter block (about 16 KB) is built in a per-thread
+    // buffer: only the words the plan uses are written
+    static thread_local std::unique_ptr<kvp::CascadeArgs> c_buf(new kvp::CascadeArgs());
+    kvp::CascadeArgs *c = c_buf.get();
     int32_t *tile_off = c->data, *mem_off = tile_off + ng + 1, *tokens = mem_off + ng + 1;
     int32_t *mem = tokens + ng, *skip = mem + nm;
     std::fill(skip, skip + S, 0);
-    const int MT = kvp::kPreRows / G;
+    const int MT = kvp::kPreQTiles * (kvp::kPreRows / G);  // members per prefix CTA
     int kt_min = INT32_MAX;
     tile_off[0] = 0;
     mem_off[0] = 0;
@@ -324,7 +327,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     c->n_members = (int32_t)nm;
     c->qk_scale = a.qk_scale;
     int P_pre = 0;
-    rc = cascade_dispatch(L.head_dim, G, nullptr, c.get(), 0, p->sm_count, nullptr, false, &P_pre);
+    rc = cascade_dispatch(L.head_dim, G, nullptr, c, 0, p->sm_count, nullptr, false, &P_pre);
     if (rc) return rc;
     // key splits: fill the GPU's CTA slots once, every split non-empty
     c->KS = std::max(1, std::min({P_pre / std::max(1, tiles * Hkv), kvp::kMaxKeySplits, kt_min}));
@@ -335,7 +338,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.KS = c->KS;
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
-    rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c.get(), tiles * Hkv * c->KS, p->sm_count,
+    rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, tiles * Hkv * c->KS, p->sm_count,
                           (cudaStream_t)stream, true, &P_pre);
     if (rc) return rc;
     return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
