@@ -463,7 +463,13 @@ int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream);
  * g = floor(h / G), G = Hq / Hkv (contiguous head groups):
  *     out[s][h] = sum_{j<n} softmax_j(scale * q[s][h] . K_j) V_j
  * with K_j, V_j the rows of head g at position j, found through dev_table.
- * q, out: bf16 [S][Hq][d] device arrays.  A sequence with n == 0 gets zeros.
+ * q, out: bf16 [S][Hq][d] arrays, 16-byte aligned, in device memory or in
+ * pinned (page-locked, mapped) host memory: the kernels read q and write
+ * out with ordinary loads and stores, which on GB300 cross the coherent
+ * NVLink-C2C link to host memory, so a caller holding a step's inputs and
+ * results on the host needs no separate copies (the same holds for k_new
+ * and v_new of the calls below).  The pool, table, lengths and workspace
+ * are device memory.  A sequence with n == 0 gets zeros.
  * Arithmetic: fp32 products and accumulation, online softmax in base 2,
  * bf16 output rounded to nearest-even.
  * Work split: the batch's KV is cut into 16-token tiles of one (sequence,

@@ -217,12 +217,39 @@ class DeviceSteps:
         self.max_blocks, self.scale, self.num_splits = max_blocks, scale, num_splits
         self.table = torch.full((rows, max_blocks), -1, dtype=torch.int32, device=dev)
         self.lens = torch.zeros(rows, dtype=torch.int32, device=dev)
-        self.q = _dev_u16(q, dev)
-        self.k_new = _dev_u16(k_new, dev)
-        self.v_new = _dev_u16(v_new, dev)
+        # q, k_new and v_new are views of one contiguous buffer, so a step's
+        # inputs reach the device with a single copy (each view stays 16-byte
+        # aligned: every part is a whole number of d-element rows, d % 8 == 0)
+        parts = [np.ascontiguousarray(a).reshape(-1) for a in (q, k_new, v_new)]
+        self.inputs = _dev_u16(np.concatenate(parts), dev)
+        sizes = [p.size for p in parts]
+        q_, k_, v_ = torch.split(self.inputs, sizes)
+        self.q = q_.view(np.shape(q))
+        self.k_new = k_.view(np.shape(k_new))
+        self.v_new = v_.view(np.shape(v_new))
         self.out = torch.empty((S, Hq, d), dtype=torch.bfloat16, device=dev)
         self.ws_bytes = K.kv_workspace_bytes(pool.handle, layout, S, Hq, max_blocks, num_splits)
         self.ws = torch.empty(max(256, self.ws_bytes), dtype=torch.uint8, device=dev)
+        self._shapes = (np.shape(q), np.shape(k_new), np.shape(v_new))
+        self._device_io = (self.inputs, self.out)
+
+    def io(self, inputs=None, out=None) -> None:
+        """Point q / k_new / v_new at `inputs` (bf16, laid out like
+        self.inputs: q, then k_new, then v_new) and the output at `out`:
+        device tensors, or pinned host tensors that the kernels read and
+        write directly over the GPU's coherent link to host memory.  With no
+        arguments, back to this batch's device buffers."""
+        if inputs is None:
+            inputs, out = self._device_io
+        if inputs.numel() != self._device_io[0].numel() or out.numel() != self._device_io[1].numel():
+            raise ValueError("io buffers must match the batch's input and output sizes")
+        if inputs.device.type == "cpu" and not (inputs.is_pinned() and out.is_pinned()):
+            raise ValueError("host io buffers must be pinned")
+        sizes = [int(np.prod(sh)) for sh in self._shapes]
+        q_, k_, v_ = torch.split(inputs.view(torch.bfloat16).reshape(-1), sizes)
+        self.inputs = inputs
+        self.q, self.k_new, self.v_new = (t.view(sh) for t, sh in zip((q_, k_, v_), self._shapes))
+        self.out = out.view(self._device_io[1].shape)
 
     def sync(self, seqtab, stream=None) -> None:
         seqtab.sync(self.table, self.lens, stream)
