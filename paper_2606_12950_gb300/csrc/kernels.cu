@@ -276,7 +276,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     int64_t nm = 0;
     for (int i = 0; i < ng; ++i) {
         const kv_prefix_group &gr = cas->groups[i];
-        if (gr.count < 1 || gr.tokens < kvp::kPreKeys || gr.tokens % kvp::kPreKeys || gr.tokens % bs ||
+        if (gr.count < 1 || gr.tokens < kvp::kPreChunk || gr.tokens % kvp::kPreChunk || gr.tokens % bs ||
             (int64_t)gr.tokens > (int64_t)max_blocks * bs)
             return KV_ERR_INVALID_ARG;
         nm += gr.count;
@@ -298,7 +298,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         tile_off[i + 1] = tile_off[i] + (gr.count + MT - 1) / MT;
         mem_off[i + 1] = mem_off[i] + gr.count;
         tokens[i] = gr.tokens;
-        kt_min = std::min(kt_min, gr.tokens / kvp::kPreKeys);
+        kt_min = std::min(kt_min, gr.tokens / kvp::kPreChunk);
         for (int j = mem_off[i]; j < mem_off[i + 1]; ++j) {
             const int32_t s = cas->members[j];
             if (s < 0 || s >= S || skip[s]) return KV_ERR_INVALID_ARG;  // each sequence in one group at most

@@ -120,6 +120,32 @@ def test_many_members_several_row_tiles_and_key_splits(G):
     assert pool.error() == 0
 
 
+@pytest.mark.parametrize("G", [4, 5])
+def test_scores_rising_inside_a_key_tile(G):
+    """The prefix's keys at tokens 64..127 and 192..255 are scaled by 8, so
+    the second 64-key half of each 128-key tile of the prefix kernel scores
+    far above the first (by more than 2^8 in base 2): the running max rises
+    inside a tile (the P already written for the tile is rescaled) and
+    between tiles (O is rescaled)."""
+    Hkv, d, bs = 2, 128, 16
+    pre = [256 + 40, 256 + 300, 256 + 7, 900]
+    groups = [([0, 1, 2], 256)]
+    b = build(4500 + G, pre, groups, G, Hkv, d, bs)
+    lead = groups[0][0][0]
+    for j in list(range(64, 128)) + list(range(192, 256)):
+        base = int(b.table[lead][j // bs]) * b.page_elems
+        for g in range(Hkv):
+            k0 = base + (g * bs + j % bs) * d  # K of head g at offset j % bs
+            row = W.bf16_bits_to_f64(b.pool[k0:k0 + d]) * 8.0
+            b.pool[k0:k0 + d] = W.bf16_bits_from_f32(row.astype(np.float32))
+    pool, db = run(b, groups)
+    ref_pool = oracle.batch_append(b)
+    assert np.array_equal(pool.download(), ref_pool)
+    ref = oracle.batch_attention(b, pool=ref_pool)
+    check(db.out_f64(), ref, f"rising scores G={G}")
+    assert pool.error() == 0
+
+
 def test_cascade_agrees_with_plain_attention():
     """Same inputs through paged_decode_attn_append and the cascade: both
     within tolerance of the oracle and within a few bf16 ulps of each other."""
