@@ -444,8 +444,8 @@ def main():
             ev_pair[0].record(stream)
         for _, buf in wl.tables():
             if cascade is not None:
-                buf.cascade(cascade, stream=stream)  # prefix kernel + attention (fused append) + combine
-                n += 3
+                buf.cascade(cascade, stream=stream)  # plan, attention (fused append), prefix kernel, combine
+                n += 4
             elif args.separate_append:
                 buf.append(stream)
                 buf.attend(stream)

@@ -3,13 +3,13 @@
 #include "attn_launch.cuh"
 
 int kvp_attn_d128(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sm_count,
-                 cudaStream_t st, bool launch, int *P_out)
+                 cudaStream_t st, int what, int *P_out)
 {
     using namespace kvp;
 #define KVP_CASE(GG)                                                                                   \
     case GG:                                                                                           \
-        return variant == 1 ? attn_run<128, GG, FmaCompute<128, GG>>(tmap, *a, P_req, sm_count, st, launch, P_out) \
-                            : attn_run<128, GG, MmaCompute<128, GG>>(tmap, *a, P_req, sm_count, st, launch, P_out);
+        return variant == 1 ? attn_run<128, GG, FmaCompute<128, GG>>(tmap, *a, P_req, sm_count, st, what, P_out) \
+                            : attn_run<128, GG, MmaCompute<128, GG>>(tmap, *a, P_req, sm_count, st, what, P_out);
     switch (G) {
         KVP_CASE(1)
         KVP_CASE(2)
@@ -17,7 +17,7 @@ int kvp_attn_d128(int variant, int G, const CUtensorMap *tmap, const kvp::AttnAr
         KVP_CASE(5)
     case 8:
         if (variant == 1) return KV_ERR_UNSUPPORTED;
-        return attn_run<128, 8, MmaCompute<128, 8>>(tmap, *a, P_req, sm_count, st, launch, P_out);
+        return attn_run<128, 8, MmaCompute<128, 8>>(tmap, *a, P_req, sm_count, st, what, P_out);
     default:
         return KV_ERR_UNSUPPORTED;
     }

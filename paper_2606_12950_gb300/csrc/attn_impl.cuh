@@ -600,8 +600,12 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     if (tid == 32) prefetch_tensormap(&tmap);
     // launched as a programmatic dependent: everything above touches only
     // this CTA; wait here for the grid before (lengths, table, pool writes)
-    grid_launch_dependents();
+    // In shared-prefix mode the dependents are released only after the wait:
+    // the prefix kernel, which follows this grid without waiting for it,
+    // relies on every CTA here having seen the grids before complete.
+    if (!a.skip) grid_launch_dependents();
     grid_dependency_wait();
+    if (a.skip) grid_launch_dependents();
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {

@@ -34,9 +34,12 @@ int cached_occupancy(Fn fn, int threads, size_t smem, int *occ)
     return KV_OK;
 }
 
+// what: kLaunchQuery (only *P_out), kLaunchBoth (attention, then combine),
+// kLaunchAttention, kLaunchCombine
+enum { kLaunchQuery = 0, kLaunchBoth = 1, kLaunchAttention = 2, kLaunchCombine = 3 };
+
 template <int D, int G, class Comp>
-int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaStream_t st, bool launch,
-             int *P_out)
+int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaStream_t st, int what, int *P_out)
 {
     auto fn = paged_attn_kernel<D, G, Comp>;
     static std::atomic<bool> attr_set{false};
@@ -51,7 +54,7 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     if (cached_occupancy(fn, kThreads, smem, &occ) != KV_OK) return KV_ERR_CUDA;
     const int P = P_req > 0 ? P_req : std::max(1, occ) * std::max(1, sm_count);
     *P_out = P;
-    if (!launch) return KV_OK;
+    if (what == kLaunchQuery) return KV_OK;
     a.rows_cap = kRowsCap;
     a.P = P;
     // both kernels are programmatic dependents of what precedes them in the
@@ -67,7 +70,8 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
+    if (what != kLaunchCombine && cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
+    if (what == kLaunchAttention) return KV_OK;
     CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv, a.skip, a.ws_pre, a.KS};
     cudaLaunchConfig_t ccfg = cfg;
     // records per run: at most P * kWarps parts spread over the runs, plus
@@ -117,9 +121,9 @@ int cascade_run(const CUtensorMap *tmap, const CascadeArgs *c, int grid, int sm_
 
 // one entry per head dim; variant 1 = CUDA cores, 2 = tensor-core MMA
 int kvp_attn_d64(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sm_count,
-                 cudaStream_t st, bool launch, int *P_out);
+                 cudaStream_t st, int what, int *P_out);
 int kvp_attn_d128(int variant, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sm_count,
-                  cudaStream_t st, bool launch, int *P_out);
+                  cudaStream_t st, int what, int *P_out);
 int kvp_cascade_d64(int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sm_count,
                     cudaStream_t st, bool launch, int *P_out);
 int kvp_cascade_d128(int G, const CUtensorMap *tmap, const kvp::CascadeArgs *c, int grid, int sm_count,

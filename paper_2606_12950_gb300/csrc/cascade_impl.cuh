@@ -183,11 +183,13 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     const uint32_t tbase = *tslot;
     bool dead = false;
     constexpr int TMA_WARP = kPreQTiles * kPreSoftWarps, MMA_WARP = TMA_WARP + 1;
+    // This grid follows the decode kernel in the stream without waiting for
+    // it: it reads only q and the block table, which the decode kernel's
+    // CTAs had all seen complete before this grid could launch.  It waits for
+    // the decode grid at its end (below), so that the combine after it sees
+    // both grids' records.
     grid_launch_dependents();
-    grid_dependency_wait();  // the table (and q) come from the grids before
-
-    if (blockIdx.x == 0)
-        for (int s = tid; s < c.S; s += kPreThreads) c.ws_skip[s] = skip[s];
+    (void)skip;
 
     // Q rows (member, head) of KV head g into the swizzled K-major layout the
     // MMA reads: softmax thread t fills row t % 128 of Q tile t / 128; rows
@@ -411,6 +413,7 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tbase, kPreQTiles * kPreTmemCols);
+    grid_dependency_wait();  // the decode grid before this one has completed
 }
 
 template <int D>

@@ -118,10 +118,36 @@ int attn_shape(const kv_pool *p, int layout, int S, int Hq, int max_blocks, int 
 }
 
 int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::AttnArgs *a, int P_req, int sms,
-             cudaStream_t st, bool launch, int *P_out)
+             cudaStream_t st, int what, int *P_out)
 {
-    if (D == 64) return kvp_attn_d64(variant, G, tmap, a, P_req, sms, st, launch, P_out);
-    return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, launch, P_out);
+    if (D == 64) return kvp_attn_d64(variant, G, tmap, a, P_req, sms, st, what, P_out);
+    return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, what, P_out);
+}
+
+// The shared-prefix plan's per-sequence skip into the workspace, where the
+// decode kernel (suffix tiles start there) and the combine read it.  It
+// waits for the previous grid first: the previous step's combine may still
+// read the old skips.
+__global__ void cascade_plan_kernel(const __grid_constant__ kvp::CascadeArgs c)
+{
+    kvp::grid_dependency_wait();
+    kvp::grid_launch_dependents();
+    const int32_t *skip = c.data + 2 * (c.n_groups + 1) + c.n_groups + c.n_members;
+    for (int s = threadIdx.x; s < c.S; s += blockDim.x) c.ws_skip[s] = skip[s];
+}
+
+int cascade_plan_run(const kvp::CascadeArgs *c, cudaStream_t st)
+{
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, cascade_plan_kernel, *c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
 // workspace: per-run (first part, parts) as int2 (padded to 256 bytes),
@@ -186,7 +212,7 @@ int kv_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int max_bloc
     a.S = S;
     a.Hkv = L.num_kv_heads;
     int P = 0;
-    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, false, &P);
+    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, kvp::kLaunchQuery, &P);
     if (rc) return rc;
     size_t off;
     *out_bytes = ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &off);
@@ -204,7 +230,7 @@ int kv_cascade_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int 
     a.S = S;
     a.Hkv = L.num_kv_heads;
     int P = 0;
-    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, 0, p->sm_count, nullptr, false, &P);
+    rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, 0, p->sm_count, nullptr, kvp::kLaunchQuery, &P);
     if (rc) return rc;
     size_t o1, o2, o3;
     *out_bytes = cascade_ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &o1, &o2, &o3);
@@ -254,7 +280,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.bs = p->desc.block_size;
     a.qk_scale = scale * 1.4426950408889634f;
     int P = 0;
-    rc = dispatch(variant, L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, false, &P);
+    rc = dispatch(variant, L.head_dim, G, nullptr, &a, num_splits, p->sm_count, nullptr, kvp::kLaunchQuery, &P);
     if (rc) return rc;
     size_t part_off;
     if (!cas) {
@@ -265,11 +291,17 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         rc = ensure_tmap(p, layout);
         if (rc) return rc;
         return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count,
-                        (cudaStream_t)stream, true, &P);
+                        (cudaStream_t)stream, kvp::kLaunchBoth, &P);
     }
 
-    // ---- shared-prefix mode: validate the plan, build the prefix kernel's
-    // parameters, then launch prefix kernel, decode kernel and combine ----
+    // ---- shared-prefix mode: validate the plan and build the prefix
+    // kernel's parameters, then launch, in stream order: the plan kernel
+    // (per-sequence skips), the decode kernel over the suffixes, the prefix
+    // kernel and the combine.  The prefix kernel does not wait for the decode
+    // kernel before it works (it reads only q and the table), so its CTAs
+    // start on SMs the decode kernel's tail frees; it waits for the decode
+    // grid at its end, so the combine, which waits for the prefix kernel,
+    // sees both grids' records ----
     const int bs = p->desc.block_size, Hkv = L.num_kv_heads;
     const int ng = cas->n_groups;
     if (ng < 1 || !cas->groups || !cas->members) return KV_ERR_INVALID_ARG;
@@ -338,11 +370,16 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.KS = c->KS;
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
+    rc = cascade_plan_run(c, (cudaStream_t)stream);
+    if (rc) return rc;
+    rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
+                  kvp::kLaunchAttention, &P);
+    if (rc) return rc;
     rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, tiles * Hkv * c->KS, p->sm_count,
                           (cudaStream_t)stream, true, &P_pre);
     if (rc) return rc;
     return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
-                    true, &P);
+                    kvp::kLaunchCombine, &P);
 }
 
 }  // namespace
