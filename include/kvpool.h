@@ -249,7 +249,10 @@ int kv_block_table_upload(kv_pool *pool, int layout, const int32_t *host_table, 
  * (a "reservation miss"), a shared prompt prefix is held by reference, and
  * blocks go back to the pool when a stage or sequence ends (§III-C).  Every
  * change is recorded so that kv_seqtab_sync sends only changed table entries
- * to the device.  Not thread-safe; one table per host thread.
+ * to the device.  Not thread-safe; one table per host thread.  A pool
+ * destroyed while tables over it are still open detaches them: their blocks
+ * end with the pool, every later call on them that would touch a slot
+ * returns KV_ERR_INVALID_ARG, and kv_seqtab_destroy only frees the table.
  */
 typedef struct kv_seqtab kv_seqtab;
 

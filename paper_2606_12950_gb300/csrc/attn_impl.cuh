@@ -56,6 +56,15 @@ constexpr int kMinUnitsPerPart = 4;
 constexpr uint32_t kHalfBytes = kTile * 128;      // one 64-column box: 16 rows x 128 B
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
+// Loads of data written by earlier grids: through L2 only (ld.global.cg) when
+// the kernel did not wait for the grid before it (shared-prefix mode), so that
+// no line an earlier kernel left in this SM's L1 is read; plain otherwise.
+template <class T>
+__device__ __forceinline__ T ld_prior(const T *p, bool l2_only)
+{
+    return l2_only ? __ldcg(p) : *p;
+}
+
 struct AttnArgs {
     const uint16_t *q;
     uint16_t *out;
@@ -132,7 +141,7 @@ struct FmaCompute {
     float p[TPG][G];
     int grp, sub, nv;
 
-    __device__ __forceinline__ void begin(const uint16_t *qrow, float qk_scale, int lane)
+    __device__ __forceinline__ void begin(const uint16_t *qrow, float qk_scale, int lane, bool l2_only)
     {
         grp = lane / LPT;
         sub = lane % LPT;
@@ -141,7 +150,7 @@ struct FmaCompute {
 #pragma unroll
             for (int j = 0; j < NCH; ++j) {
                 const int c = sub + j * LPT;
-                uint4 w = *reinterpret_cast<const uint4 *>(qrow + h * D + c * 8);
+                uint4 w = ld_prior(reinterpret_cast<const uint4 *>(qrow + h * D + c * 8), l2_only);
                 uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
@@ -306,7 +315,7 @@ struct MmaCompute {
     float qk_scale;
     int gid, tig, lane_, nv;
 
-    __device__ __forceinline__ void begin(const uint16_t *qrow, float scale, int lane)
+    __device__ __forceinline__ void begin(const uint16_t *qrow, float scale, int lane, bool l2_only)
     {
         lane_ = lane;
         gid = lane >> 2;
@@ -315,8 +324,10 @@ struct MmaCompute {
 #pragma unroll
         for (int kk = 0; kk < KS; ++kk) {
             if (gid < G) {
-                qf[kk][0] = *reinterpret_cast<const uint32_t *>(qrow + gid * D + kk * 16 + tig * 2);
-                qf[kk][1] = *reinterpret_cast<const uint32_t *>(qrow + gid * D + kk * 16 + tig * 2 + 8);
+                qf[kk][0] = ld_prior(reinterpret_cast<const unsigned int *>(qrow + gid * D + kk * 16 + tig * 2),
+                                     l2_only);
+                qf[kk][1] = ld_prior(reinterpret_cast<const unsigned int *>(qrow + gid * D + kk * 16 + tig * 2 + 8),
+                                     l2_only);
             } else {
                 qf[kk][0] = 0u;
                 qf[kk][1] = 0u;
@@ -465,40 +476,41 @@ struct Piece {
     int32_t skip;          // leading tokens handled by the prefix kernel
 };
 
-__device__ __forceinline__ int32_t clamp_len(const AttnArgs &a, int s, bool report_errors)
+// Context length of sequence s, read once per CTA in the prologue and clamped
+// to the table's reach with the error reported.
+__device__ __forceinline__ int32_t load_len(const AttnArgs &a, int s, int32_t *raw_out)
 {
-    int32_t n = a.ctx_lens[s];
+    const int32_t raw = ld_prior(a.ctx_lens + s, a.skip != nullptr);
     const int32_t cap = a.max_blocks * a.bs;
-    if (n < 0 || n > cap) {
-        if (report_errors) report(a.err, KV_ERR_DEVICE_BOUNDS);
-        n = n < 0 ? 0 : cap;
+    *raw_out = raw;
+    if (raw < 0 || raw > cap) {
+        report(a.err, KV_ERR_DEVICE_BOUNDS);
+        return raw < 0 ? 0 : cap;
     }
-    return n;
+    return raw;
 }
 
 // leading tokens of sequence s (context n) left to the prefix kernel: 0
-// outside cascade mode; a value that is not a multiple of 16 in [0, n] is
-// reported and clamped
-__device__ __forceinline__ int32_t seq_skip(const AttnArgs &a, int s, int32_t n, bool report_errors)
+// outside shared-prefix mode; a value that is not a multiple of 16 in
+// [0, n] is reported and clamped
+__device__ __forceinline__ int32_t load_skip(const AttnArgs &a, int s, int32_t n)
 {
     if (!a.skip) return 0;
-    int32_t k = a.skip[s];
+    int32_t k = __ldcg(a.skip + s);
     if (k < 0 || k > n || (k % kTile)) {
-        if (report_errors) report(a.err, KV_ERR_DEVICE_BOUNDS);
+        report(a.err, KV_ERR_DEVICE_BOUNDS);
         k = k < 0 ? 0 : (k > n ? n : k);
         k -= k % kTile;
     }
     return k;
 }
 
-// units of sequence s: 16-token tiles of its (suffix) context, per KV head
-__device__ __forceinline__ int32_t seq_units(const AttnArgs &a, int s, bool report_errors, int32_t *ne_out)
-{
-    const int32_t n = clamp_len(a, s, report_errors);
-    const int32_t ne = n - seq_skip(a, s, n, report_errors);
-    if (ne_out) *ne_out = ne;
-    return ((ne + kTile - 1) / kTile) * a.Hkv;
-}
+// The CTA's copy of the per-sequence values, after T[0 .. S]: NL[s] = the
+// clamped length, with bit 31 set when the stored length was out of range;
+// SK[s] = the clamped skip.
+__device__ __forceinline__ int32_t seq_len(const int32_t *T, int S, int s) { return T[S + 1 + s] & 0x7fffffff; }
+__device__ __forceinline__ bool seq_len_clamped(const int32_t *T, int S, int s) { return T[S + 1 + s] < 0; }
+__device__ __forceinline__ int32_t seq_skip(const int32_t *T, int S, int s) { return T[2 * S + 1 + s]; }
 
 // largest s with T[s] <= u; T[s] = first unit of sequence s, T[S] = total,
 // so empty sequences (T[s] == T[s+1]) are skipped
@@ -519,8 +531,8 @@ __device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T
     const int32_t g = (u - T[s]) / nt;
     p.s = s;
     p.g = g;
-    p.n = clamp_len(a, s, false);
-    p.skip = seq_skip(a, s, p.n, false);
+    p.n = seq_len(T, a.S, s);
+    p.skip = seq_skip(T, a.S, s);
     p.run_begin = T[s] + g * nt;
     p.run_end = p.run_begin + nt;
     p.pb = u;
@@ -535,8 +547,8 @@ __device__ __forceinline__ int32_t unit_row(const AttnArgs &a, const int32_t *T,
     const int32_t nt = (T[s + 1] - T[s]) / a.Hkv;
     const int32_t within = u - T[s];
     const int32_t g = within / nt;
-    const int32_t tok0 = seq_skip(a, s, clamp_len(a, s, false), false) + (within - g * nt) * kTile;
-    const int32_t phys = a.table[(int64_t)s * a.max_blocks + tok0 / a.bs];
+    const int32_t tok0 = seq_skip(T, a.S, s) + (within - g * nt) * kTile;
+    const int32_t phys = ld_prior(a.table + (int64_t)s * a.max_blocks + tok0 / a.bs, a.skip != nullptr);
     if (phys < 0 || (int64_t)phys + a.pages_per_block > a.pool_pages) return -1;
     return (int32_t)((int64_t)phys * a.rows_per_page + (tok0 % a.bs) + (int64_t)g * a.bs);
 }
@@ -588,7 +600,9 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kWarps * STAGE_BYTES);  // K[w], V[w]
     int32_t *misc = reinterpret_cast<int32_t *>(bars + 2 * kWarps);                     // [16] scratch
     int32_t *T = misc + 16;                                                              // [S + 1]
-    int32_t *rows = T + a.S + 1;                                                         // [rows_cap]
+    int32_t *NL = T + a.S + 1;                                                           // [S]
+    int32_t *SK = NL + a.S;                                                              // [S]
+    int32_t *rows = SK + a.S;                                                            // [rows_cap]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int S = a.S, Hkv = a.Hkv, Hq = a.Hkv * G;
@@ -598,14 +612,18 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         fence_mbar_init();
     }
     if (tid == 32) prefetch_tensormap(&tmap);
-    // launched as a programmatic dependent: everything above touches only
-    // this CTA; wait here for the grid before (lengths, table, pool writes)
-    // In shared-prefix mode the dependents are released only after the wait:
-    // the prefix kernel, which follows this grid without waiting for it,
-    // relies on every CTA here having seen the grids before complete.
-    if (!a.skip) grid_launch_dependents();
-    grid_dependency_wait();
-    if (a.skip) grid_launch_dependents();
+    // Launched as a programmatic dependent: everything above touches only
+    // this CTA.  Outside shared-prefix mode, wait here for the grid before
+    // (lengths, table, pool writes).  In shared-prefix mode the grid before
+    // is the prefix kernel, which released this grid only after its own wait
+    // had seen every earlier grid complete (plan, table sync, the previous
+    // step's combine); this grid does not wait for the prefix kernel here,
+    // so the two run side by side on disjoint SMs, and waits for it at its
+    // end (cascade_done), so that the combine after it sees both grids'
+    // records.  Data from earlier grids is then read through L2 (ld_prior).
+    grid_launch_dependents();
+    if (!a.skip) grid_dependency_wait();
+    const bool cascade_done = a.skip != nullptr;
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {
@@ -613,16 +631,21 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         const int lo = min(S, tid * per), hi = min(S, lo + per);
         int32_t local = 0;
         for (int s = lo; s < hi; ++s) {
-            int32_t ne;
-            local += seq_units(a, s, true, &ne);
+            int32_t raw;
+            const int32_t n = load_len(a, s, &raw);
+            const int32_t k = load_skip(a, s, n);
+            NL[s] = n | (raw != n ? (int32_t)0x80000000 : 0);
+            SK[s] = k;
+            const int32_t ne = n - k;
+            local += ((ne + kTile - 1) / kTile) * Hkv;
             // the fused append needs the new token outside a shared prefix
-            if (ne == 0 && a.skip && a.k_new && clamp_len(a, s, false) > 0 && (s % a.P) == (int)blockIdx.x)
+            if (ne == 0 && a.skip && a.k_new && n > 0 && (s % a.P) == (int)blockIdx.x)
                 report(a.err, KV_ERR_DEVICE_BOUNDS);
             if (ne == 0 && (s % a.P) == (int)blockIdx.x) {
                 // an empty context has no softmax: its output is defined as
                 // zero; a sequence whose whole context is a shared prefix
                 // gets its output from the prefix records alone
-                if (clamp_len(a, s, false) == 0)
+                if (n == 0)
                     for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
                 for (int g = 0; g < Hkv; ++g) a.ws_run[(int64_t)s * Hkv + g] = make_int2(0, 0);
             }
@@ -638,9 +661,9 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         int32_t base = 0;
         for (int w = 0; w < warp; ++w) base += misc[w];
         int32_t run = base + incl - local;
-        for (int s = lo; s < hi; ++s) {
+        for (int s = lo; s < hi; ++s) {  // this thread's own NL / SK entries
             T[s] = run;
-            run += seq_units(a, s, false, nullptr);
+            run += ((seq_len(T, S, s) - seq_skip(T, S, s) + kTile - 1) / kTile) * Hkv;
         }
         if (tid == 0) {
             int32_t tot = 0;
@@ -660,7 +683,10 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     const int64_t np_min = W > 0 ? (W / kMinUnitsPerPart > 0 ? W / kMinUnitsPerPart : 1) : 0;
     const int64_t NP = np_min < (int64_t)a.P * kWarps ? np_min : (int64_t)a.P * kWarps;
     const int64_t first_part = (int64_t)blockIdx.x * kWarps;
-    if (first_part >= NP) return;
+    if (first_part >= NP) {
+        if (cascade_done) grid_dependency_wait();
+        return;
+    }
     const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
     const int32_t cu0 = (int32_t)(first_part * W / NP);                             // this CTA's units
     const int32_t cu1 = (int32_t)(last_part * W / NP);
@@ -674,7 +700,10 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     }
 
     const int64_t part = first_part + warp;
-    if (part >= NP) return;  // no CTA-wide barrier below this point
+    if (part >= NP) {  // no CTA-wide barrier below this point
+        if (cascade_done) grid_dependency_wait();
+        return;
+    }
     const int32_t u0 = (int32_t)(part * W / NP);
     const int32_t u1 = (int32_t)((part + 1) * W / NP);
 
@@ -696,20 +725,20 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         Piece pc;
         decode_piece(a, T, u, u1, pc);
         Comp comp;
-        comp.begin(a.q + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D, a.qk_scale, lane);
+        comp.begin(a.q + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D, a.qk_scale, lane, cascade_done);
         for (int32_t uu = pc.pb; uu < pc.pe; ++uu) {
             const uint32_t par = consumed & 1u;
             const int nvalid = min(kTile, pc.n - pc.skip - (uu - pc.run_begin) * kTile);
             const bool more = uu + 1 < u1;
             // fused append: the run's last tile holds position n-1, whose K/V
             // row is this step's new token; this warp alone reads that tile
-            const bool app = a.k_new != nullptr && uu == pc.run_end - 1 && a.ctx_lens[pc.s] == pc.n;
+            const bool app = a.k_new != nullptr && uu == pc.run_end - 1 && !seq_len_clamped(T, S, pc.s);
             const int arow = (pc.n - 1) % kTile;
             wait_phase(bk, par, a.err, dead);
             if (app) {
                 if (lane < D / 8)
-                    *reinterpret_cast<uint4 *>(Ks + swz(arow, lane)) = *reinterpret_cast<const uint4 *>(
-                        a.k_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8);
+                    *reinterpret_cast<uint4 *>(Ks + swz(arow, lane)) = ld_prior(reinterpret_cast<const uint4 *>(
+                        a.k_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8), cascade_done);
                 __syncwarp();
             }
             comp.qk(Ks, nvalid);
@@ -721,8 +750,8 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             wait_phase(bv, par, a.err, dead);
             if (app) {
                 if (lane < D / 8)
-                    *reinterpret_cast<uint4 *>(Vs + swz(arow, lane)) = *reinterpret_cast<const uint4 *>(
-                        a.v_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8);
+                    *reinterpret_cast<uint4 *>(Vs + swz(arow, lane)) = ld_prior(reinterpret_cast<const uint4 *>(
+                        a.v_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8), cascade_done);
                 __syncwarp();
             }
             comp.pv(Vs);
@@ -735,7 +764,8 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
                     const int which = lane / (D / 8), c = lane % (D / 8);
                     const int64_t row = (int64_t)y + arow + (int64_t)which * Hkv * a.bs;
                     const uint16_t *src = (which ? a.v_new : a.k_new) + ((int64_t)pc.s * Hkv + pc.g) * D + c * 8;
-                    *reinterpret_cast<uint4 *>(a.pool + row * D + c * 8) = *reinterpret_cast<const uint4 *>(src);
+                    *reinterpret_cast<uint4 *>(a.pool + row * D + c * 8) =
+                        ld_prior(reinterpret_cast<const uint4 *>(src), cascade_done);
                 }
             }
             fence_proxy_async_smem();
@@ -757,6 +787,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             a.ws_run[r] = make_int2(p_first, split ? p_last - p_first + 1 : 0);
         u = pc.pe;
     }
+    if (cascade_done) grid_dependency_wait();
 }
 
 // ------------------------------------------------------------ combine ---
@@ -891,7 +922,7 @@ template <int D, int G>
 inline size_t attn_smem_bytes(int S, int rows_cap)
 {
     const size_t stage = 2ull * (D / 64) * kHalfBytes;
-    return 1024 + (size_t)kWarps * stage + (2 * kWarps) * 8 + 64 + (size_t)(S + 1) * 4 + (size_t)rows_cap * 4;
+    return 1024 + (size_t)kWarps * stage + (2 * kWarps) * 8 + 64 + (size_t)(3 * S + 1) * 4 + (size_t)rows_cap * 4;
 }
 
 // partial records: one per (run, part) pair that a run can touch

@@ -183,11 +183,11 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     const uint32_t tbase = *tslot;
     bool dead = false;
     constexpr int TMA_WARP = kPreQTiles * kPreSoftWarps, MMA_WARP = TMA_WARP + 1;
-    // This grid follows the decode kernel in the stream without waiting for
-    // it: it reads only q and the block table, which the decode kernel's
-    // CTAs had all seen complete before this grid could launch.  It waits for
-    // the decode grid at its end (below), so that the combine after it sees
-    // both grids' records.
+    // Wait for the grid before (the plan kernel; through it the table sync
+    // and the previous step's combine), then release the decode kernel that
+    // follows: it runs beside this grid on the SMs this grid leaves free and
+    // relies on this wait having completed in every CTA here.
+    grid_dependency_wait();
     grid_launch_dependents();
     (void)skip;
 
@@ -413,7 +413,6 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     __syncthreads();
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tbase, kPreQTiles * kPreTmemCols);
-    grid_dependency_wait();  // the decode grid before this one has completed
 }
 
 template <int D>

@@ -296,12 +296,11 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
 
     // ---- shared-prefix mode: validate the plan and build the prefix
     // kernel's parameters, then launch, in stream order: the plan kernel
-    // (per-sequence skips), the decode kernel over the suffixes, the prefix
-    // kernel and the combine.  The prefix kernel does not wait for the decode
-    // kernel before it works (it reads only q and the table), so its CTAs
-    // start on SMs the decode kernel's tail frees; it waits for the decode
-    // grid at its end, so the combine, which waits for the prefix kernel,
-    // sees both grids' records ----
+    // (per-sequence skips), the prefix kernel, the decode kernel over the
+    // suffixes and the combine.  The prefix kernel takes about a quarter of
+    // the SMs (one CTA each); the decode kernel, sized to the SMs left, runs
+    // beside it without waiting for it and waits for it at its end, so the
+    // combine, which waits for the decode grid, sees both grids' records ----
     const int bs = p->desc.block_size, Hkv = L.num_kv_heads;
     const int ng = cas->n_groups;
     if (ng < 1 || !cas->groups || !cas->members) return KV_ERR_INVALID_ARG;
@@ -361,8 +360,22 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     int P_pre = 0;
     rc = cascade_dispatch(L.head_dim, G, nullptr, c, 0, p->sm_count, nullptr, false, &P_pre);
     if (rc) return rc;
-    // key splits: fill the GPU's CTA slots once, every split non-empty
-    c->KS = std::max(1, std::min({P_pre / std::max(1, tiles * Hkv), kvp::kMaxKeySplits, kt_min}));
+    // key splits: as many as keep the prefix grid within a quarter of the
+    // GPU's CTA slots for it (at least one; every split non-empty)
+    const int pre_slots = std::max(1, P_pre / 4);
+    c->KS = std::max(1, std::min({pre_slots / std::max(1, tiles * Hkv), kvp::kMaxKeySplits, kt_min}));
+    // the decode grid fills the SMs the prefix grid leaves free (all of them
+    // when the prefix grid needs more than half the GPU: the decode CTAs then
+    // start as prefix CTAs finish)
+    const int pre_ctas = tiles * Hkv * c->KS;
+    const int pre_occ = std::max(1, P_pre / std::max(1, p->sm_count));
+    const int pre_sms = (pre_ctas + pre_occ - 1) / pre_occ;
+    const int free_sms = 2 * pre_sms <= p->sm_count ? p->sm_count - pre_sms : p->sm_count;
+    if (num_splits <= 0) {
+        rc = dispatch(variant, L.head_dim, G, nullptr, &a, 0, free_sms, nullptr, kvp::kLaunchQuery, &P);
+        if (rc) return rc;
+        num_splits = P;
+    }
     a.ws_run = reinterpret_cast<int2 *>(ws);
     a.ws_part = reinterpret_cast<float *>(ws + part_off);
     a.skip = c->ws_skip;
@@ -372,11 +385,11 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     if (rc) return rc;
     rc = cascade_plan_run(c, (cudaStream_t)stream);
     if (rc) return rc;
+    rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, pre_ctas, p->sm_count, (cudaStream_t)stream, true,
+                          &P_pre);
+    if (rc) return rc;
     rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                   kvp::kLaunchAttention, &P);
-    if (rc) return rc;
-    rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, tiles * Hkv * c->KS, p->sm_count,
-                          (cudaStream_t)stream, true, &P_pre);
     if (rc) return rc;
     return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                     kvp::kLaunchCombine, &P);

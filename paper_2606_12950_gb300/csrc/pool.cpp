@@ -119,6 +119,12 @@ int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool)
 int kv_pool_destroy(kv_pool *pool)
 {
     if (!pool) return KV_ERR_INVALID_ARG;
+    {
+        // sequence tables still open lose their pool: their blocks end with it
+        std::lock_guard<std::mutex> g(pool->mu);
+        for (kv_seqtab *t : pool->seqtabs) kvp_seqtab_detach(t);
+        pool->seqtabs.clear();
+    }
     if (pool->vmm.active) kvp_vmm_release_all(pool);
     delete pool;
     return KV_OK;

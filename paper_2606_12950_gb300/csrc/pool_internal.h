@@ -52,6 +52,7 @@ struct kv_pool {
     bool tmap_ok[KV_MAX_LAYOUTS] = {false, false, false, false};
     kv_vmm_state vmm;
     uint64_t shuffle_state = 0;               // splitmix64 state for placing newly mapped superpages
+    std::vector<kv_seqtab *> seqtabs;         // live sequence tables over this pool (detached on destroy)
     std::mutex mu;
 };
 
@@ -59,6 +60,10 @@ struct kv_pool {
 int kvp_vmm_map_chunk(kv_pool *p);                  // map the next unmapped chunk
 int kvp_vmm_unmap_chunk(kv_pool *p, int64_t chunk);  // unmap a chunk whose superpages are all free
 void kvp_vmm_release_all(kv_pool *p);                // on destroy
+
+// Called by kv_pool_destroy, with the pool's mutex held, for every sequence
+// table still open over the pool (seqtab.cpp).
+void kvp_seqtab_detach(kv_seqtab *t);
 
 // Validate that a block id is a whole block of layout L inside the pool.
 // In a VMM pool the block must also lie in a mapped chunk.

@@ -15,7 +15,8 @@
 
 namespace {
 
-bool slot_ok(const kv_seqtab *t, int s) { return t && s >= 0 && s < t->S; }
+// a table whose pool was destroyed first is detached (pool == nullptr)
+bool slot_ok(const kv_seqtab *t, int s) { return t && t->pool && s >= 0 && s < t->S; }
 
 void set_entry(kv_seqtab *t, int s, int i, int32_t v)
 {
@@ -28,6 +29,8 @@ void set_entry(kv_seqtab *t, int s, int i, int32_t v)
 }
 
 }  // namespace
+
+void kvp_seqtab_detach(kv_seqtab *t) { t->pool = nullptr; }
 
 extern "C" {
 
@@ -49,6 +52,10 @@ int kv_seqtab_create(kv_pool *pool, int layout, int max_seqs, int max_blocks, kv
     t->pending.assign((size_t)max_seqs * max_blocks, 0);
     t->full_dirty = true;
     std::memset(&t->counters, 0, sizeof t->counters);
+    {
+        std::lock_guard<std::mutex> g(pool->mu);
+        pool->seqtabs.push_back(t);
+    }
     *out = t;
     return KV_OK;
 }
@@ -73,11 +80,15 @@ int kv_seqtab_destroy(kv_seqtab *t)
 {
     if (!t) return KV_ERR_INVALID_ARG;
     int rc = KV_OK;
-    for (int s = 0; s < t->S; ++s)
-        if (t->held[(size_t)s] > 0) {
-            int r = kv_seq_release(t, s);
-            if (r && !rc) rc = r;
-        }
+    if (kv_pool *pool = t->pool) {
+        for (int s = 0; s < t->S; ++s)
+            if (t->held[(size_t)s] > 0) {
+                int r = kv_seq_release(t, s);
+                if (r && !rc) rc = r;
+            }
+        std::lock_guard<std::mutex> g(pool->mu);
+        pool->seqtabs.erase(std::remove(pool->seqtabs.begin(), pool->seqtabs.end(), t), pool->seqtabs.end());
+    }
     delete t;
     return rc;
 }
@@ -124,7 +135,7 @@ int kv_seq_set_len(kv_seqtab *t, int s, int32_t len)
 
 int kv_seq_advance(kv_seqtab *t, int n, const int32_t *seqs, int32_t *n_grown)
 {
-    if (!t || (seqs && n < 0)) return KV_ERR_INVALID_ARG;
+    if (!t || !t->pool || (seqs && n < 0)) return KV_ERR_INVALID_ARG;
     std::vector<int32_t> list;
     if (seqs) {
         list.assign(seqs, seqs + n);

@@ -122,3 +122,26 @@ def test_shared_prefix_survives_release_of_its_origin():
     with pytest.raises(K.KVError):
         t.share_prefix(1, 2, 1)  # source holds nothing
     t.close()
+
+
+def test_destroying_the_pool_first_detaches_its_tables():
+    # tables closed after their pool (garbage-collection order) must not touch
+    # the freed pool: they are detached and only free themselves
+    pool, t = make(S=4, max_blocks=8)
+    t.reserve(0, 64)
+    t.set_len(0, 64)
+    t2 = K.SeqTab(pool, 0, 2, 8)
+    t2.reserve(1, 16)
+    K.kv_pool_destroy(pool)
+    for call in (lambda: t.reserve(1, 16), lambda: t.advance(), lambda: t.release(0), lambda: t2.trim(1)):
+        with pytest.raises(K.KVError) as e:
+            call()
+        assert e.value.code == K.KV_ERR_INVALID_ARG
+    t.close()
+    t2.close()
+    # a table destroyed before its pool unregisters itself
+    pool, t = make(S=2, max_blocks=4)
+    t.reserve(0, 16)
+    t.close()
+    assert K.kv_pool_stats(pool)["blocks_used"][0] == 0
+    K.kv_pool_destroy(pool)
