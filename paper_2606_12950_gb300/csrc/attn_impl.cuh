@@ -141,7 +141,8 @@ struct FmaCompute {
     float p[TPG][G];
     int grp, sub, nv;
 
-    __device__ __forceinline__ void begin(const uint16_t *qrow, float qk_scale, int lane, bool l2_only)
+    // qrow: the run's G query rows, staged in shared memory
+    __device__ __forceinline__ void begin(const uint16_t *qrow, float qk_scale, int lane)
     {
         grp = lane / LPT;
         sub = lane % LPT;
@@ -150,7 +151,7 @@ struct FmaCompute {
 #pragma unroll
             for (int j = 0; j < NCH; ++j) {
                 const int c = sub + j * LPT;
-                uint4 w = ld_prior(reinterpret_cast<const uint4 *>(qrow + h * D + c * 8), l2_only);
+                uint4 w = *reinterpret_cast<const uint4 *>(qrow + h * D + c * 8);
                 uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
@@ -315,7 +316,8 @@ struct MmaCompute {
     float qk_scale;
     int gid, tig, lane_, nv;
 
-    __device__ __forceinline__ void begin(const uint16_t *qrow, float scale, int lane, bool l2_only)
+    // qrow: the run's G query rows, staged in shared memory
+    __device__ __forceinline__ void begin(const uint16_t *qrow, float scale, int lane)
     {
         lane_ = lane;
         gid = lane >> 2;
@@ -324,10 +326,8 @@ struct MmaCompute {
 #pragma unroll
         for (int kk = 0; kk < KS; ++kk) {
             if (gid < G) {
-                qf[kk][0] = ld_prior(reinterpret_cast<const unsigned int *>(qrow + gid * D + kk * 16 + tig * 2),
-                                     l2_only);
-                qf[kk][1] = ld_prior(reinterpret_cast<const unsigned int *>(qrow + gid * D + kk * 16 + tig * 2 + 8),
-                                     l2_only);
+                qf[kk][0] = *reinterpret_cast<const uint32_t *>(qrow + gid * D + kk * 16 + tig * 2);
+                qf[kk][1] = *reinterpret_cast<const uint32_t *>(qrow + gid * D + kk * 16 + tig * 2 + 8);
             } else {
                 qf[kk][0] = 0u;
                 qf[kk][1] = 0u;
@@ -596,8 +596,11 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     extern __shared__ uint8_t smem_raw[];
     // stages need 1024-byte alignment for the 128-byte swizzle pattern
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    constexpr uint32_t QB = G * D * 2, AB = 2 * D * 2;  // q rows of a run; its new K and V rows
     uint8_t *stages = smem;                                                              // [kWarps][STAGE]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kWarps * STAGE_BYTES);  // K[w], V[w]
+    uint8_t *qbufs = stages + (size_t)kWarps * STAGE_BYTES;                              // [kWarps][QB]
+    uint8_t *abufs = qbufs + (size_t)kWarps * QB;                                        // [kWarps][AB]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(abufs + (size_t)kWarps * AB);          // K[w], V[w]
     int32_t *misc = reinterpret_cast<int32_t *>(bars + 2 * kWarps);                     // [16] scratch
     int32_t *T = misc + 16;                                                              // [S + 1]
     int32_t *NL = T + a.S + 1;                                                           // [S]
@@ -717,6 +720,19 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         issue_half<D>(&tmap, a, T, rows, cu0, u0, 0, k_addr, bk, policy);
         issue_half<D>(&tmap, a, T, rows, cu0, u0, 1, v_addr, bv, policy);
     }
+    // A run's q rows and, for the run's last tile, its new K/V rows are staged
+    // in this warp's shared buffers by cp.async one piece ahead, so that no
+    // piece start or append waits on a dependent global load.
+    uint8_t *qb = qbufs + (size_t)warp * QB;
+    uint8_t *ab = abufs + (size_t)warp * AB;
+    const uint32_t qb_addr = smem_u32(qb), ab_addr = smem_u32(ab);
+    {
+        const int s0 = find_seq(T, S, u0);
+        const int32_t nt0 = (T[s0 + 1] - T[s0]) / Hkv;
+        const uint16_t *src = a.q + ((int64_t)s0 * Hq + (int64_t)((u0 - T[s0]) / nt0) * G) * D;
+        for (uint32_t c = lane; c < QB / 16; c += 32) cp_async16(qb_addr + c * 16, src + c * 8);
+        cp_async_commit();
+    }
 
     bool dead = false;
     uint32_t consumed = 0;
@@ -724,21 +740,37 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     while (u < u1) {
         Piece pc;
         decode_piece(a, T, u, u1, pc);
+        cp_async_wait_all();  // this piece's q rows
+        __syncwarp();
         Comp comp;
-        comp.begin(a.q + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D, a.qk_scale, lane, cascade_done);
+        comp.begin(reinterpret_cast<const uint16_t *>(qb), a.qk_scale, lane);
+        __syncwarp();  // every lane holds its q fragments: the buffer may be refilled
+        // fused append: the run's last tile holds position n-1, whose K/V row
+        // is this step's new token; this warp alone reads that tile
+        const bool app_run = a.k_new != nullptr && pc.pe == pc.run_end && !seq_len_clamped(T, S, pc.s);
+        if (app_run && lane < AB / 16) {
+            const int which = lane / (D / 8), c = lane % (D / 8);
+            cp_async16(ab_addr + lane * 16, (which ? a.v_new : a.k_new) + ((int64_t)pc.s * Hkv + pc.g) * D + c * 8);
+        }
+        if (pc.pe < u1) {  // the next piece's q rows
+            const int s2 = find_seq(T, S, pc.pe);
+            const int32_t nt2 = (T[s2 + 1] - T[s2]) / Hkv;
+            const uint16_t *src = a.q + ((int64_t)s2 * Hq + (int64_t)((pc.pe - T[s2]) / nt2) * G) * D;
+            for (uint32_t c = lane; c < QB / 16; c += 32) cp_async16(qb_addr + c * 16, src + c * 8);
+        }
+        cp_async_commit();
         for (int32_t uu = pc.pb; uu < pc.pe; ++uu) {
             const uint32_t par = consumed & 1u;
             const int nvalid = min(kTile, pc.n - pc.skip - (uu - pc.run_begin) * kTile);
             const bool more = uu + 1 < u1;
-            // fused append: the run's last tile holds position n-1, whose K/V
-            // row is this step's new token; this warp alone reads that tile
-            const bool app = a.k_new != nullptr && uu == pc.run_end - 1 && !seq_len_clamped(T, S, pc.s);
+            const bool app = app_run && uu == pc.run_end - 1;
             const int arow = (pc.n - 1) % kTile;
             wait_phase(bk, par, a.err, dead);
             if (app) {
+                cp_async_wait_all();  // the new K/V rows
+                __syncwarp();
                 if (lane < D / 8)
-                    *reinterpret_cast<uint4 *>(Ks + swz(arow, lane)) = ld_prior(reinterpret_cast<const uint4 *>(
-                        a.k_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8), cascade_done);
+                    *reinterpret_cast<uint4 *>(Ks + swz(arow, lane)) = *reinterpret_cast<const uint4 *>(ab + lane * 16);
                 __syncwarp();
             }
             comp.qk(Ks, nvalid);
@@ -750,8 +782,8 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             wait_phase(bv, par, a.err, dead);
             if (app) {
                 if (lane < D / 8)
-                    *reinterpret_cast<uint4 *>(Vs + swz(arow, lane)) = ld_prior(reinterpret_cast<const uint4 *>(
-                        a.v_new + ((int64_t)pc.s * Hkv + pc.g) * D + lane * 8), cascade_done);
+                    *reinterpret_cast<uint4 *>(Vs + swz(arow, lane)) =
+                        *reinterpret_cast<const uint4 *>(ab + D * 2 + lane * 16);
                 __syncwarp();
             }
             comp.pv(Vs);
@@ -760,12 +792,11 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
                 // the tile have completed, and no other unit covers that row
                 const int32_t k = uu - cu0;
                 const int32_t y = k < a.rows_cap ? rows[k] : unit_row(a, T, uu);
-                if (y >= 0 && lane < D / 4) {
+                if (y >= 0 && lane < AB / 16) {
                     const int which = lane / (D / 8), c = lane % (D / 8);
                     const int64_t row = (int64_t)y + arow + (int64_t)which * Hkv * a.bs;
-                    const uint16_t *src = (which ? a.v_new : a.k_new) + ((int64_t)pc.s * Hkv + pc.g) * D + c * 8;
                     *reinterpret_cast<uint4 *>(a.pool + row * D + c * 8) =
-                        ld_prior(reinterpret_cast<const uint4 *>(src), cascade_done);
+                        *reinterpret_cast<const uint4 *>(ab + lane * 16);
                 }
             }
             fence_proxy_async_smem();
@@ -922,7 +953,9 @@ template <int D, int G>
 inline size_t attn_smem_bytes(int S, int rows_cap)
 {
     const size_t stage = 2ull * (D / 64) * kHalfBytes;
-    return 1024 + (size_t)kWarps * stage + (2 * kWarps) * 8 + 64 + (size_t)(3 * S + 1) * 4 + (size_t)rows_cap * 4;
+    const size_t bufs = (size_t)G * D * 2 + 2 * D * 2;  // per warp: q rows, new K/V rows
+    return 1024 + (size_t)kWarps * (stage + bufs) + (2 * kWarps) * 8 + 64 + (size_t)(3 * S + 1) * 4 +
+           (size_t)rows_cap * 4;
 }
 
 // partial records: one per (run, part) pair that a run can touch

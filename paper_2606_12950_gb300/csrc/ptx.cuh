@@ -93,6 +93,15 @@ __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map)
 
 // Programmatic dependent launch: wait until the preceding grid in the stream
 // has completed and its memory is visible; allow the next grid to launch.
+// 16-byte asynchronous copy global -> shared through L2 only (cp.async.cg),
+// grouped by commit and awaited by wait_all; no registers hold the data.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 __device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void grid_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" :::); }
 
