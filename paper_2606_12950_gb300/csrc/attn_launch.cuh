@@ -78,7 +78,7 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     // the prefix records in shared-prefix mode
     const double per_run = (double)P * kWarps / std::max(1, a.S * a.Hkv) + 1.0 + (a.skip ? a.KS : 0);
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv));
-    ccfg.blockDim = dim3((unsigned)(combine_groups<D, G>(per_run) * (G * D / 4)));
+    ccfg.blockDim = dim3((unsigned)(combine_groups<D, G>(per_run, a.skip != nullptr) * (G * D / 4)));
     ccfg.dynamicSmemBytes = 0;
     if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G>, c) != cudaSuccess) return KV_ERR_CUDA;
     return KV_OK;
