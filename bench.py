@@ -18,6 +18,7 @@ Prints one JSON line on rank 0.
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -458,6 +459,15 @@ def main():
         launches_per_step = n
         return nbytes
 
+    # No garbage-collector pass inside the timed regions: a full pass over the
+    # interpreter's objects (torch's included) stalled the submitting thread
+    # for 3.4 ms in one measured step, long enough to drain the GPU's queue.
+    # Everything alive now is moved out of the collector's view, and
+    # collection is off until both timed regions are done.
+    gc.collect()
+    gc.freeze()
+    gc.disable()
+
     # the clock sampler starts first; the warm-up steps then run right before
     # the timed region, so the GPU enters it busy rather than after an idle gap
     clocks = ClockSampler(local)
@@ -526,6 +536,7 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
+    gc.enable()
     for buf in bufs:
         buf.io()
     ms, e2e_ms, tot = aggregate_ranks(dist, torch.device("cuda", local), ms, e2e_ms,

@@ -120,6 +120,25 @@ def test_many_members_several_row_tiles_and_key_splits(G):
     assert pool.error() == 0
 
 
+def test_prefix_grid_larger_than_half_the_gpu():
+    """700 sharers at G = 4, Hkv = 8: 11 row tiles x 8 KV heads = 88 prefix
+    CTAs, more than half of the SMs, so the decode grid is sized to the
+    whole GPU and its CTAs start as prefix CTAs finish."""
+    rng = np.random.default_rng(4300)
+    n = 700
+    pre = (128 + rng.integers(0, 200, size=n)).tolist() + [90, 333]
+    groups = [(list(range(n)), 128)]
+    b = build(4300, pre, groups, 4, 8, 128, 16)
+    pool, db = run(b, groups)
+    ref_pool = oracle.batch_append(b)
+    assert np.array_equal(pool.download(), ref_pool)
+    ids = np.array(sorted(set(rng.choice(len(pre), 24, replace=False).tolist()) | {0, n - 1, n, n + 1}), np.int32)
+    ref = oracle.paged_attention(ref_pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q, b.table, b.ctx_lens,
+                                 b.scale, seq_ids=ids)
+    check(db.out_f64()[ids], ref[ids], "700 sharers")
+    assert pool.error() == 0
+
+
 @pytest.mark.parametrize("G", [4, 5])
 def test_scores_rising_inside_a_key_tile(G):
     """The prefix's keys at tokens 64..127 and 192..255 are scaled by 8, so
