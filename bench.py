@@ -389,6 +389,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
+    ap.add_argument("--separate-sync", action="store_true",
+                    help="table sync with its own kernel instead of carried by the decode launch")
     ap.add_argument("--pool", default="fixed", choices=["fixed", "vmm"],
                     help="llama8b: a fixed device buffer, or the VMM-backed elastic pool")
     ap.add_argument("--no-cascade", action="store_true",
@@ -432,19 +434,31 @@ def main():
         for _, buf in wl.tables():
             buf.use_cascade()
 
+    fuse_sync = cascade is None and not args.separate_append and not args.separate_sync
+
+    def sync_kernels():
+        return sum(tab.counters()["sync_launches"] for tab, _ in wl.tables() if tab is not None)
+
     def step(ev_pair=None):
         """host bookkeeping, table sync, then append + attention per batch"""
         nonlocal launches_per_step
         nbytes = wl.host_step()
         n = 0
-        for tab, buf in wl.tables():
-            if tab is not None:
-                tab.sync(buf.table, buf.lens, stream)
-                n += 1
+        if not fuse_sync:
+            for tab, buf in wl.tables():
+                if tab is not None:
+                    tab.sync(buf.table, buf.lens, stream)
+                    n += 1
         if ev_pair is not None:
             ev_pair[0].record(stream)
-        for _, buf in wl.tables():
-            if cascade is not None:
+        for tab, buf in wl.tables():
+            if fuse_sync and tab is not None:
+                # table sync, append and attention: the decode launch carries
+                # the sync when it fits (else a sync kernel runs first; those
+                # launches are counted from the tables' counters)
+                buf.sync_append_attend(tab, stream)
+                n += 2
+            elif cascade is not None:
                 buf.cascade(cascade, stream=stream)  # plan, attention (fused append), prefix kernel, combine
                 n += 4
             elif args.separate_append:
@@ -487,12 +501,14 @@ def main():
     if dist:
         dist.barrier()
     step_bytes = []
+    sync0 = sync_kernels()
     h0 = time.perf_counter()
     t_start.record(stream)
     for i in range(args.steps):
         step_bytes.append(step(evs[i // SAMPLE] if i % SAMPLE == 0 else None))
     t_end.record(stream)
     host_us = (time.perf_counter() - h0) * 1e6 / args.steps  # host submission time per step
+    extra_sync_launches = sync_kernels() - sync0 if fuse_sync else 0
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
@@ -566,6 +582,7 @@ def main():
     config = {"workload": wl.name, **wl.config, "num_splits": args.num_splits, "variant": args.variant,
               "pool": args.pool if args.workload == "llama8b" else "fixed",
               "append": "separate kernel" if args.separate_append else "fused into attention",
+              "table_sync": ("carried by the decode launch when it fits" if fuse_sync else "separate kernel"),
               "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
                                 else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,
               "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
@@ -582,7 +599,7 @@ def main():
                                                                  "attention call in the timed region"},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": launches_per_step * args.steps + extra_sync_launches,
         "host_us_per_step": host_us,
         "host_cores": pinned_cores,
         "clocks": clk,

@@ -506,6 +506,25 @@ int paged_decode_attn_append(kv_pool *pool, int layout, const uint16_t *q, const
                              int num_splits, void *workspace, size_t ws_bytes, void *stream);
 
 /*
+ * kv_seqtab_sync(t, dev_table, dev_ctx_lens, stream) followed by
+ * paged_decode_attn_append (k_new, v_new given) or paged_decode_attn (both
+ * NULL) over the table's first S rows, with layout and max_blocks taken from
+ * the table, in one launch when it fits: when the table's lengths and its
+ * changed entries since the last sync make at most 128 words, they travel
+ * as parameters of the decode kernel, which reads them from there and
+ * writes them to dev_ctx_lens / dev_table for later kernels (the separate
+ * sync kernel, its hand-off and a dependent read of the lengths drop out of
+ * the step).  Otherwise (the first sync, larger batches or many changes)
+ * the call runs kv_seqtab_sync and then the plain call.  Results, device
+ * table and lengths afterwards are those of the two calls; errors are theirs
+ * (KV_ERR_INVALID_ARG also when t is not over `pool` or S > max_seqs).
+ */
+int paged_decode_attn_seqtab(kv_pool *pool, kv_seqtab *t, const uint16_t *q, const uint16_t *k_new,
+                             const uint16_t *v_new, uint16_t *out, int32_t *dev_table, int32_t *dev_ctx_lens,
+                             int S, int Hq, float scale, int num_splits, void *workspace, size_t ws_bytes,
+                             void *stream);
+
+/*
  * Shared-prefix ("cascade") decode attention.  Sequences that hold the same
  * physical blocks at the start of their block tables -- a system prompt
  * shared by reference by every stage of an agent workflow (§III-B, §III-C)

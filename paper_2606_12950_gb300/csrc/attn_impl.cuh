@@ -65,6 +65,12 @@ __device__ __forceinline__ T ld_prior(const T *p, bool l2_only)
     return l2_only ? __ldcg(p) : *p;
 }
 
+// Words of a table sync carried by the decode kernel's parameters (lengths,
+// then (flat index, value) pairs of changed table entries): 512 bytes, which
+// every launch carries.  A 1.8 KB block cost the launch more than the
+// separate sync kernel saved (measured on config 2).
+constexpr int kSyncWords = 128;
+
 struct AttnArgs {
     const uint16_t *q;
     uint16_t *out;
@@ -92,6 +98,15 @@ struct AttnArgs {
     const int32_t *skip;
     const float *ws_pre;
     int32_t KS;
+    // fused table sync (paged_decode_attn_seqtab): this step's lengths of
+    // rows [0, sync_nlens) and its changed table entries travel here.  The
+    // kernel takes the lengths and those entries from here, and the CTAs
+    // write them to sync_lens / sync_table for later kernels.  Null: none.
+    int32_t *sync_table;
+    int32_t *sync_lens;
+    int32_t sync_nlens;
+    int32_t sync_npatch;
+    int32_t sync_words[kSyncWords];
 };
 
 __device__ __forceinline__ void report(int32_t *err, int code) { atomicCAS(err, 0, code); }
@@ -480,7 +495,7 @@ struct Piece {
 // to the table's reach with the error reported.
 __device__ __forceinline__ int32_t load_len(const AttnArgs &a, int s, int32_t *raw_out)
 {
-    const int32_t raw = ld_prior(a.ctx_lens + s, a.skip != nullptr);
+    const int32_t raw = a.sync_table ? a.sync_words[s] : ld_prior(a.ctx_lens + s, a.skip != nullptr);
     const int32_t cap = a.max_blocks * a.bs;
     *raw_out = raw;
     if (raw < 0 || raw > cap) {
@@ -539,6 +554,18 @@ __device__ __forceinline__ void decode_piece(const AttnArgs &a, const int32_t *T
     p.pe = p.run_end < u1 ? p.run_end : u1;
 }
 
+// Block table entry idx (flat): this step's value when the table sync is
+// fused into the launch and changed that entry, else the table's.
+__device__ __forceinline__ int32_t table_entry(const AttnArgs &a, int64_t idx)
+{
+    if (a.sync_table) {
+        const int32_t *pw = a.sync_words + a.sync_nlens;
+        for (int j = 0; j < a.sync_npatch; ++j)
+            if (pw[2 * j] == idx) return pw[2 * j + 1];
+    }
+    return ld_prior(a.table + idx, a.skip != nullptr);
+}
+
 // Pool row of unit u's K tile (TMA y coordinate; V is Hkv*bs rows further),
 // or -1 if the block table names a block outside the pool.
 __device__ __forceinline__ int32_t unit_row(const AttnArgs &a, const int32_t *T, int32_t u)
@@ -548,7 +575,7 @@ __device__ __forceinline__ int32_t unit_row(const AttnArgs &a, const int32_t *T,
     const int32_t within = u - T[s];
     const int32_t g = within / nt;
     const int32_t tok0 = seq_skip(T, a.S, s) + (within - g * nt) * kTile;
-    const int32_t phys = ld_prior(a.table + (int64_t)s * a.max_blocks + tok0 / a.bs, a.skip != nullptr);
+    const int32_t phys = table_entry(a, (int64_t)s * a.max_blocks + tok0 / a.bs);
     if (phys < 0 || (int64_t)phys + a.pages_per_block > a.pool_pages) return -1;
     return (int32_t)((int64_t)phys * a.rows_per_page + (tok0 % a.bs) + (int64_t)g * a.bs);
 }
@@ -627,6 +654,14 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     grid_launch_dependents();
     if (!a.skip) grid_dependency_wait();
     const bool cascade_done = a.skip != nullptr;
+    if (a.sync_table) {
+        // fused table sync: the grids before have completed (the wait
+        // above), and no CTA of this grid reads what is written here
+        const int stride = a.P * kThreads, i0 = (int)blockIdx.x * kThreads + tid;
+        for (int i = i0; i < a.sync_nlens; i += stride) a.sync_lens[i] = a.sync_words[i];
+        const int32_t *pw = a.sync_words + a.sync_nlens;
+        for (int j = i0; j < a.sync_npatch; j += stride) a.sync_table[pw[2 * j]] = pw[2 * j + 1];
+    }
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {

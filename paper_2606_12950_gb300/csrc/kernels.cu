@@ -10,6 +10,7 @@
 
 #include "attn_launch.cuh"
 #include "pool_internal.h"
+#include "seqtab_internal.h"
 
 namespace {
 
@@ -247,10 +248,17 @@ struct CascadePlan {
     const int32_t *members;
 };
 
+// a host sequence table whose pending changes travel with the decode launch
+struct FusedSync {
+    kv_seqtab *t;
+    int32_t *dev_table;
+    int32_t *dev_lens;
+};
+
 int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
               uint16_t *out, const int32_t *dev_table, const int32_t *dev_ctx_lens, int max_blocks, int S, int Hq,
               float scale, int num_splits, void *workspace, size_t ws_bytes, void *stream,
-              const CascadePlan *cas = nullptr)
+              const CascadePlan *cas = nullptr, const FusedSync *sync = nullptr)
 {
     int G = 0;
     if (num_splits < 0 || !std::isfinite(scale)) return KV_ERR_INVALID_ARG;
@@ -290,8 +298,29 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(workspace) + part_off);
         rc = ensure_tmap(p, layout);
         if (rc) return rc;
-        return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count,
-                        (cudaStream_t)stream, kvp::kLaunchBoth, &P);
+        if (sync) {
+            // the caller checked that the lengths and changed entries fit
+            kv_seqtab *t = sync->t;
+            const int nl = t->S, np = (int)t->changed.size();
+            a.sync_table = sync->dev_table;
+            a.sync_lens = sync->dev_lens;
+            a.sync_nlens = nl;
+            a.sync_npatch = np;
+            for (int i = 0; i < nl; ++i) a.sync_words[i] = t->lens[(size_t)i];
+            for (int j = 0; j < np; ++j) {
+                const int32_t idx = t->changed[(size_t)j];
+                a.sync_words[nl + 2 * j] = idx;
+                a.sync_words[nl + 2 * j + 1] = t->table[(size_t)idx];
+            }
+        }
+        rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
+                      kvp::kLaunchBoth, &P);
+        if (rc || !sync) return rc;
+        kv_seqtab *t = sync->t;
+        t->counters.entries_uploaded += (int64_t)t->changed.size();
+        for (int32_t idx : t->changed) t->pending[(size_t)idx] = 0;
+        t->changed.clear();
+        return KV_OK;
     }
 
     // ---- shared-prefix mode: validate the plan and build the prefix
@@ -415,6 +444,26 @@ int paged_decode_attn_append(kv_pool *p, int layout, const uint16_t *q, const ui
     if (!k_new || !v_new) return KV_ERR_INVALID_ARG;
     return attn_call(p, layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale,
                      num_splits, workspace, ws_bytes, stream);
+}
+
+int paged_decode_attn_seqtab(kv_pool *p, kv_seqtab *t, const uint16_t *q, const uint16_t *k_new,
+                             const uint16_t *v_new, uint16_t *out, int32_t *dev_table, int32_t *dev_ctx_lens, int S,
+                             int Hq, float scale, int num_splits, void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!p || !t || t->pool != p || !dev_table || !dev_ctx_lens || S < 0 || S > t->S) return KV_ERR_INVALID_ARG;
+    if ((!k_new) != (!v_new)) return KV_ERR_INVALID_ARG;
+    const size_t words = (size_t)t->S + 2 * t->changed.size();
+    if (t->full_dirty || words > (size_t)kvp::kSyncWords || S == 0) {
+        // too much to carry with the launch (or nothing to launch): the
+        // separate sync kernel (or a whole-table copy), then the plain call
+        int rc = kv_seqtab_sync(t, dev_table, dev_ctx_lens, stream);
+        if (rc) return rc;
+        return attn_call(p, t->layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, t->max_blocks, S, Hq, scale,
+                         num_splits, workspace, ws_bytes, stream);
+    }
+    const FusedSync sync{t, dev_table, dev_ctx_lens};
+    return attn_call(p, t->layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, t->max_blocks, S, Hq, scale,
+                     num_splits, workspace, ws_bytes, stream, nullptr, &sync);
 }
 
 }  // extern "C"

@@ -169,6 +169,7 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn": [P, I, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
             "paged_decode_attn_append": [P, I, P, P, P, P, P, P, I, I, I, F, I, P, SZ, P],
+            "paged_decode_attn_seqtab": [P, P, P, P, P, P, P, P, I, I, F, I, P, SZ, P],
             "kv_set_attn_variant": [P, I],
             "kv_cascade_workspace_bytes": [P, I, I, I, I, ctypes.POINTER(SZ)],
             "kv_pool_create_vmm": [ctypes.POINTER(kv_pool_desc), ctypes.POINTER(kv_vmm_desc), ctypes.POINTER(P)],
@@ -417,6 +418,17 @@ def paged_decode_attn_append(pool, layout: int, q, k_new, v_new, out, dev_table,
                                           _addr(dev_table), _addr(dev_ctx_lens), int(max_blocks), int(S),
                                           int(Hq), float(scale), int(num_splits), _addr(workspace),
                                           int(ws_bytes), _stream(stream)))
+
+
+def paged_decode_attn_seqtab(pool, seqtab, q, k_new, v_new, out, dev_table, dev_ctx_lens, S: int, Hq: int,
+                             scale: float, num_splits: int, workspace, ws_bytes: int, stream=None) -> None:
+    """kv_seqtab_sync + paged_decode_attn(_append) in one launch when the
+    table's lengths and changed entries fit the decode kernel's parameters."""
+    h = seqtab.handle if isinstance(seqtab, SeqTab) else seqtab
+    _check("paged_decode_attn_seqtab",
+           lib().paged_decode_attn_seqtab(pool, h, _addr(q), _addr(k_new), _addr(v_new), _addr(out),
+                                          _addr(dev_table), _addr(dev_ctx_lens), int(S), int(Hq), float(scale),
+                                          int(num_splits), _addr(workspace), int(ws_bytes), _stream(stream)))
 
 
 def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_blocks: int, S: int,

@@ -259,6 +259,13 @@ class DeviceSteps:
                                    self.table, self.lens, self.max_blocks, self.S, self.Hq, self.scale,
                                    self.num_splits, self.ws, self.ws.numel(), stream)
 
+    def sync_append_attend(self, seqtab, stream=None) -> None:
+        """seqtab's table sync, the append and the attention: one launch of
+        the decode kernel (plus the combine) when the sync fits in it."""
+        K.paged_decode_attn_seqtab(self.pool.handle, seqtab, self.q, self.k_new, self.v_new, self.out, self.table,
+                                   self.lens, self.S, self.Hq, self.scale, self.num_splits, self.ws, self.ws.numel(),
+                                   stream)
+
     def append(self, stream=None) -> None:
         K.kv_append(self.pool.handle, self.layout, self.k_new, self.v_new, self.table, self.lens,
                     self.max_blocks, self.S, stream)

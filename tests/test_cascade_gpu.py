@@ -120,6 +120,27 @@ def test_many_members_several_row_tiles_and_key_splits(G):
     assert pool.error() == 0
 
 
+def test_cascade_block_placement_does_not_change_bits():
+    """Moving every physical block (prefix and suffixes) to another place in
+    the pool, with the table renamed to match, gives bit-identical outputs:
+    the prefix records and their merge depend only on logical positions."""
+    pre = [256 + 1, 256 + 70, 256 + 700, 300, 256 + 33]
+    groups = [([0, 1, 2, 4], 256)]
+    b = build(4400, pre, groups, 4, 4, 128, 16, extra_blocks=40)
+    _, db1 = run(b, groups)
+    out1 = db1.out_bits()
+    rng = np.random.default_rng(5)
+    perm = rng.permutation(b.n_pages)
+    blocks = b.pool.reshape(b.n_pages, b.page_elems)
+    pool2 = np.empty_like(blocks)
+    pool2[perm] = blocks
+    b2 = build(4400, pre, groups, 4, 4, 128, 16, extra_blocks=40)
+    b2.pool = pool2.reshape(-1)
+    b2.table = np.where(b.table >= 0, perm[np.maximum(b.table, 0)], -1).astype(np.int32)
+    _, db2 = run(b2, groups)
+    assert np.array_equal(out1, db2.out_bits())
+
+
 def test_prefix_grid_larger_than_half_the_gpu():
     """700 sharers at G = 4, Hkv = 8: 11 row tiles x 8 KV heads = 88 prefix
     CTAs, more than half of the SMs, so the decode grid is sized to the

@@ -55,3 +55,63 @@ def test_sync_matches_host_after_every_change(S, max_blocks):
     assert c["sync_launches"] >= 30
     t.close()
     pool.close()
+
+
+@pytest.mark.parametrize("S", [24, 300])
+def test_fused_sync_gives_the_bits_of_sync_then_attention(S):
+    """paged_decode_attn_seqtab against kv_seqtab_sync followed by
+    paged_decode_attn_append, on two pools with the same contents driven by
+    the same table operations: after every step the outputs, the pools (with
+    the appended rows), the device tables and the lengths are bit-identical.
+    The steps cover launches that carry the sync (few changes), the separate
+    sync kernel (many changes, or more rows than the parameters hold) and the
+    first whole-table copy."""
+    from paper_2606_12950_gb300.runner import DevicePool, DeviceSteps
+
+    Hq, Hkv, d, bs, max_blocks = 8, 2, 128, 16, 12
+    n_pages = S * max_blocks + 8
+    page_elems = 2 * Hkv * bs * d
+    rng = np.random.default_rng(77)
+    host_pool = (rng.standard_normal(n_pages * page_elems).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    q = (rng.standard_normal((S, Hq, d)).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    kn = (rng.standard_normal((S, Hkv, d)).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    vn = (rng.standard_normal((S, Hkv, d)).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    sides = []
+    for _ in range(2):
+        pool = DevicePool(n_pages, page_elems * 2, bs, [(Hkv, d)], shuffle_seed=3)
+        pool.upload(host_pool)
+        t = K.SeqTab(pool.handle, 0, S, max_blocks)
+        buf = DeviceSteps(pool, 0, S, S, Hq, Hkv, d, max_blocks, d ** -0.5, q, kn, vn)
+        sides.append((pool, t, buf))
+    ops = np.random.default_rng(S)
+    for s in range(S):
+        tokens = int(ops.integers(1, 6 * bs))
+        for _, t, _ in sides:
+            t.reserve(s, tokens + 2 * bs)
+            t.set_len(s, tokens)
+    for step in range(12):
+        if step == 6:  # many changes at once: the separate sync kernel
+            for s in range(0, S, 2):
+                for _, t, _ in sides:
+                    t.release(s)
+                    t.reserve(s, 3 * bs)
+                    t.set_len(s, 2 * bs - 1)
+        for _, t, _ in sides:
+            tab, lens = t.host()
+            t.advance([s for s in range(S) if lens[s] + 1 < max_blocks * bs])
+        pool_a, t_a, buf_a = sides[0]
+        t_a.sync(buf_a.table, buf_a.lens)
+        buf_a.append_attend()
+        pool_b, t_b, buf_b = sides[1]
+        buf_b.sync_append_attend(t_b)
+        torch.cuda.synchronize()
+        assert np.array_equal(buf_a.out.cpu().view(torch.int16).numpy(), buf_b.out.cpu().view(torch.int16).numpy()), step
+        assert np.array_equal(buf_a.table.cpu().numpy(), buf_b.table.cpu().numpy()), step
+        assert np.array_equal(buf_a.lens.cpu().numpy(), buf_b.lens.cpu().numpy()), step
+        assert np.array_equal(pool_a.download(), pool_b.download()), step
+        tab, lens = t_b.host()
+        assert np.array_equal(buf_b.table.cpu().numpy(), tab) and np.array_equal(buf_b.lens.cpu().numpy(), lens)
+        assert pool_a.error() == 0 and pool_b.error() == 0
+    for pool, t, _ in sides:
+        t.close()
+        pool.close()
