@@ -546,9 +546,11 @@ int paged_decode_attn_seqtab(kv_pool *pool, kv_seqtab *t, const uint16_t *q, con
  * block).  A member whose length equals tokens (no append) attends over the
  * prefix alone.  A sequence is in at most one group; sequences in no group
  * are computed as by paged_decode_attn.  n_groups = 0 is paged_decode_attn
- * (or _append).  The plan travels as kernel parameters:
+ * (or _append).  The plan travels as a kernel's parameters and then in
+ * the workspace:
  *     3 * n_groups + 2 + (members) + S <= 4080 words.
- * Workspace: kv_cascade_workspace_bytes() (256-byte aligned).
+ * Workspace: kv_cascade_workspace_bytes() (256-byte aligned); nothing in it
+ * needs initialising.
  * Errors: KV_ERR_INVALID_ARG (bad plan, duplicate member, words over the
  * limit), KV_ERR_WORKSPACE, KV_ERR_UNSUPPORTED, KV_ERR_CUDA; on the device a
  * member shorter than its prefix sets KV_ERR_DEVICE_BOUNDS in the error word.

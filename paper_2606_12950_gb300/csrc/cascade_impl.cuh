@@ -37,7 +37,7 @@ constexpr int kPreSoftWarps = 4;          // per Q tile: one thread per query ro
 constexpr int kPreThreads = (kPreQTiles * kPreSoftWarps + 2) * 32;  // + TMA warp + MMA warp
 constexpr int kPreRowsCap = 256;          // 16-token sub-tiles resolved up front
 constexpr int kMaxKeySplits = 8;
-constexpr int kCascadeWords = 4080;       // plan words carried as kernel parameters
+constexpr int kCascadeWords = 4080;       // most plan words (the plan kernel's parameters, then the workspace)
 // TMEM per Q tile: S [0, 128) fp32, P over S's first 64 columns (bf16 pairs), O [128, 128 + d)
 constexpr uint32_t kPreTmemCols = 256;
 
@@ -59,9 +59,11 @@ struct CascadeArgs {
     int32_t n_members;
     float qk_scale;       // scale * log2(e)
     int32_t pad;
-    // [n_groups + 1] first row tile of each group | [n_groups + 1] first member
-    // index | [n_groups] prefix tokens | [n_members] member sequences | [S] skip
-    int32_t data[kCascadeWords];
+    // the plan in the workspace, written by the plan kernel before this grid
+    // reads it: [n_groups + 1] first row tile of each group | [n_groups + 1]
+    // first member index | [n_groups] prefix tokens | [n_members] member
+    // sequences | [S] skip
+    const int32_t *plan;
 };
 
 // members per CTA: whole query-head groups of consecutive members in each of
@@ -139,24 +141,6 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     const int g = bid % c.Hkv;
     const int tile = bid / c.Hkv;
 
-    const int32_t *tile_off = c.data;
-    const int32_t *mem_off = tile_off + c.n_groups + 1;
-    const int32_t *tokens = mem_off + c.n_groups + 1;
-    const int32_t *members = tokens + c.n_groups;
-    const int32_t *skip = members + c.n_members;
-    int grp = 0;
-    while (grp + 1 < c.n_groups && tile_off[grp + 1] <= tile) ++grp;
-    const int m0 = mem_off[grp] + (tile - tile_off[grp]) * MT;  // this CTA's members [m0, m1)
-    const int m1 = min(m0 + MT, mem_off[grp + 1]);
-    const int lead = members[mem_off[grp]];
-    const int ch_all = tokens[grp] / kPreChunk;                  // 64-key chunks of the prefix
-    const int ch0 = ks * ch_all / c.KS, ch1 = (ks + 1) * ch_all / c.KS;  // non-empty: KS <= ch_all
-    const int nch = ch1 - ch0;
-    const int nt = (nch + 1) / 2;                                // key tiles; the last may hold one chunk
-    const int nsub = nch * CSUB;
-    // valid keys of key tile t: 128, or 64 for a final half tile
-    auto tile_keys = [&](int t) { return min(kPreKeys, (nch - 2 * t) * kPreChunk); };
-
     if (tid == 0) {
         for (int i = 0; i < kPreStages; ++i) {
             mbar_init(bar(FULL + i), 1);
@@ -186,10 +170,29 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     // Wait for the grid before (the plan kernel; through it the table sync
     // and the previous step's combine), then release the decode kernel that
     // follows: it runs beside this grid on the SMs this grid leaves free and
-    // relies on this wait having completed in every CTA here.
+    // relies on this wait having completed in every CTA here.  The plan is
+    // read only after the wait: the plan kernel wrote it.
     grid_dependency_wait();
     grid_launch_dependents();
-    (void)skip;
+
+    const int32_t *tile_off = c.plan;
+    const int32_t *mem_off = tile_off + c.n_groups + 1;
+    const int32_t *tokens = mem_off + c.n_groups + 1;
+    const int32_t *members = tokens + c.n_groups;
+    // (through L2: another kernel wrote the plan)
+    int grp = 0;
+    while (grp + 1 < c.n_groups && __ldcg(tile_off + grp + 1) <= tile) ++grp;
+    const int mo = __ldcg(mem_off + grp);
+    const int m0 = mo + (tile - __ldcg(tile_off + grp)) * MT;  // this CTA's members [m0, m1)
+    const int m1 = min(m0 + MT, __ldcg(mem_off + grp + 1));
+    const int lead = __ldcg(members + mo);
+    const int ch_all = __ldcg(tokens + grp) / kPreChunk;        // 64-key chunks of the prefix
+    const int ch0 = ks * ch_all / c.KS, ch1 = (ks + 1) * ch_all / c.KS;  // non-empty: KS <= ch_all
+    const int nch = ch1 - ch0;
+    const int nt = (nch + 1) / 2;                                // key tiles; the last may hold one chunk
+    const int nsub = nch * CSUB;
+    // valid keys of key tile t: 128, or 64 for a final half tile
+    auto tile_keys = [&](int t) { return min(kPreKeys, (nch - 2 * t) * kPreChunk); };
 
     // Q rows (member, head) of KV head g into the swizzled K-major layout the
     // MMA reads: softmax thread t fills row t % 128 of Q tile t / 128; rows
@@ -199,7 +202,8 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     const int mrow = m0 + qa_tile * MQ + r / G;               // its member index
     const bool row_ok = tid < SOFT_THREADS && r < MQ * G && mrow < m1;
     if (tid < SOFT_THREADS) {
-        const uint16_t *qrow = row_ok ? c.q + ((int64_t)members[mrow] * Hq + (int64_t)g * G + r % G) * D : nullptr;
+        const uint16_t *qrow = row_ok ? c.q + ((int64_t)__ldcg(members + mrow) * Hq + (int64_t)g * G + r % G) * D
+                                      : nullptr;
         uint8_t *qdst = smem + L::Q_OFF + qa_tile * L::Q_TILE;
         uint4 qv[D / 8];
 #pragma unroll
@@ -390,7 +394,7 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
         // ---- this CTA's record per (sharer, KV head) ----
         wait_phase(o_done(a), (uint32_t)(nt - 1) & 1u, c.err, dead);
         tc_fence_after();
-        float *rec = row_ok ? c.ws_pre + (((int64_t)ks * c.S + members[mrow]) * c.Hkv + g) * MF : nullptr;
+        float *rec = row_ok ? c.ws_pre + (((int64_t)ks * c.S + __ldcg(members + mrow)) * c.Hkv + g) * MF : nullptr;
         const int hl = r % G;
         uint32_t v[32];
 #pragma unroll

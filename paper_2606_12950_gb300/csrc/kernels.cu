@@ -4,6 +4,7 @@
 #include <cmath>
 #include <memory>
 #include <mutex>
+#include <vector>
 
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -125,20 +126,44 @@ int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::Attn
     return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, what, P_out);
 }
 
-// The shared-prefix plan's per-sequence skip into the workspace, where the
-// decode kernel (suffix tiles start there) and the combine read it.  It
-// waits for the previous grid first: the previous step's combine may still
-// read the old skips.
-__global__ void cascade_plan_kernel(const __grid_constant__ kvp::CascadeArgs c)
+// The shared-prefix plan, carried as this kernel's parameters, into the
+// workspace: the whole plan for the prefix kernel, and the per-sequence
+// skips (its last S words) where the decode kernel (suffix tiles start
+// there) and the combine read them.  It waits for the previous grid first:
+// the previous step's kernels may still read the old plan and skips.  The
+// parameter block comes in two sizes so that a small plan does not pay for
+// copying the largest one into every launch (host and device time).
+template <int W>
+struct PlanParams {
+    int32_t *ws_plan;
+    int32_t *ws_skip;
+    int32_t n_words;
+    int32_t S;
+    int32_t words[W];
+};
+
+template <int W>
+__global__ void cascade_plan_kernel(const __grid_constant__ PlanParams<W> p)
 {
     kvp::grid_dependency_wait();
     kvp::grid_launch_dependents();
-    const int32_t *skip = c.data + 2 * (c.n_groups + 1) + c.n_groups + c.n_members;
-    for (int s = threadIdx.x; s < c.S; s += blockDim.x) c.ws_skip[s] = skip[s];
+    for (int i = threadIdx.x; i < p.n_words; i += blockDim.x) p.ws_plan[i] = p.words[i];
+    const int32_t *skip = p.words + (p.n_words - p.S);
+    for (int s = threadIdx.x; s < p.S; s += blockDim.x) p.ws_skip[s] = skip[s];
 }
 
-int cascade_plan_run(const kvp::CascadeArgs *c, cudaStream_t st)
+constexpr int kPlanSmallWords = 1024;
+
+template <int W>
+int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip, cudaStream_t st)
 {
+    static thread_local std::unique_ptr<PlanParams<W>> buf(new PlanParams<W>());
+    PlanParams<W> *p = buf.get();
+    p->ws_plan = ws_plan;
+    p->ws_skip = ws_skip;
+    p->n_words = n_words;
+    p->S = S;
+    std::copy(words, words + n_words, p->words);
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -148,7 +173,14 @@ int cascade_plan_run(const kvp::CascadeArgs *c, cudaStream_t st)
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, cascade_plan_kernel, *c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    return cudaLaunchKernelEx(&cfg, cascade_plan_kernel<W>, *p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+}
+
+int cascade_plan_run(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip, cudaStream_t st)
+{
+    if (n_words <= kPlanSmallWords)
+        return cascade_plan_launch<kPlanSmallWords>(words, n_words, S, ws_plan, ws_skip, st);
+    return cascade_plan_launch<kvp::kCascadeWords>(words, n_words, S, ws_plan, ws_skip, st);
 }
 
 // workspace: per-run (first part, parts) as int2 (padded to 256 bytes),
@@ -162,11 +194,13 @@ size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
 
 // cascade workspace: the above, then the per-sequence skip (padded to 256
 // bytes), then kMaxKeySplits prefix records per (sequence, KV head)
-size_t cascade_ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off, size_t *skip_off, size_t *pre_off)
+size_t cascade_ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off, size_t *skip_off, size_t *pre_off,
+                         size_t *plan_off)
 {
     const size_t base = (ws_layout(S, Hkv, G, D, P, part_off) + 255) / 256 * 256;
     *skip_off = base;
-    *pre_off = base + ((size_t)S * 4 + 255) / 256 * 256;
+    *plan_off = base + ((size_t)S * 4 + 255) / 256 * 256;
+    *pre_off = *plan_off + ((size_t)kvp::kCascadeWords * 4 + 255) / 256 * 256;
     return *pre_off + (size_t)kvp::kMaxKeySplits * S * Hkv * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
 
@@ -233,8 +267,8 @@ int kv_cascade_workspace_bytes(const kv_pool *p, int layout, int S, int Hq, int 
     int P = 0;
     rc = dispatch(pick_variant(p, G), L.head_dim, G, nullptr, &a, 0, p->sm_count, nullptr, kvp::kLaunchQuery, &P);
     if (rc) return rc;
-    size_t o1, o2, o3;
-    *out_bytes = cascade_ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &o1, &o2, &o3);
+    size_t o1, o2, o3, o4;
+    *out_bytes = cascade_ws_layout(S, L.num_kv_heads, G, L.head_dim, P, &o1, &o2, &o3, &o4);
     return KV_OK;
 }
 
@@ -342,11 +376,14 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         nm += gr.count;
     }
     if (nm > S || 2 * (ng + 1) + ng + nm + S > kvp::kCascadeWords) return KV_ERR_INVALID_ARG;
-    // the plan's parameter block (about 16 KB) is built in a per-thread
-    // buffer: only the words the plan uses are written
-    static thread_local std::unique_ptr<kvp::CascadeArgs> c_buf(new kvp::CascadeArgs());
-    kvp::CascadeArgs *c = c_buf.get();
-    int32_t *tile_off = c->data, *mem_off = tile_off + ng + 1, *tokens = mem_off + ng + 1;
+    // the plan's words are built in a per-thread buffer; the plan kernel
+    // carries them to the workspace
+    static thread_local std::vector<int32_t> words_buf;
+    const int n_words = (int)(2 * (ng + 1) + ng + nm + S);
+    words_buf.resize((size_t)n_words);
+    kvp::CascadeArgs cargs{};
+    kvp::CascadeArgs *c = &cargs;
+    int32_t *tile_off = words_buf.data(), *mem_off = tile_off + ng + 1, *tokens = mem_off + ng + 1;
     int32_t *mem = tokens + ng, *skip = mem + nm;
     std::fill(skip, skip + S, 0);
     const int MT = kvp::kPreQTiles * (kvp::kPreRows / G);  // members per prefix CTA
@@ -367,8 +404,8 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         }
     }
     const int tiles = tile_off[ng];
-    size_t skip_off, pre_off;
-    const size_t need = cascade_ws_layout(S, Hkv, G, L.head_dim, P, &part_off, &skip_off, &pre_off);
+    size_t skip_off, pre_off, plan_off;
+    const size_t need = cascade_ws_layout(S, Hkv, G, L.head_dim, P, &part_off, &skip_off, &pre_off, &plan_off);
     if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
     uint8_t *ws = reinterpret_cast<uint8_t *>(workspace);
     c->q = q;
@@ -376,6 +413,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     c->err = p->desc.device_error;
     c->ws_pre = reinterpret_cast<float *>(ws + pre_off);
     c->ws_skip = reinterpret_cast<int32_t *>(ws + skip_off);
+    c->plan = reinterpret_cast<const int32_t *>(ws + plan_off);
     c->rows_per_page = a.rows_per_page;
     c->pool_pages = a.pool_pages;
     c->pages_per_block = a.pages_per_block;
@@ -412,7 +450,8 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.KS = c->KS;
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
-    rc = cascade_plan_run(c, (cudaStream_t)stream);
+    rc = cascade_plan_run(words_buf.data(), n_words, S, reinterpret_cast<int32_t *>(ws + plan_off), c->ws_skip,
+                          (cudaStream_t)stream);
     if (rc) return rc;
     rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, pre_ctas, p->sm_count, (cudaStream_t)stream, true,
                           &P_pre);
