@@ -389,6 +389,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
+    ap.add_argument("--separate-batches", action="store_true",
+                    help="one call per co-located batch instead of one paged_decode_attn_multi call")
     ap.add_argument("--separate-sync", action="store_true",
                     help="table sync with its own kernel instead of carried by the decode launch")
     ap.add_argument("--pool", default="fixed", choices=["fixed", "vmm"],
@@ -435,6 +437,9 @@ def main():
             buf.use_cascade()
 
     fuse_sync = cascade is None and not args.separate_append and not args.separate_sync
+    # co-located batches without host tables (the same step repeated): one call
+    multi = (cascade is None and not args.separate_append and not args.separate_batches
+             and len(wl.tables()) > 1 and all(tab is None for tab, _ in wl.tables()))
 
     def sync_kernels():
         return sum(tab.counters()["sync_launches"] for tab, _ in wl.tables() if tab is not None)
@@ -451,7 +456,11 @@ def main():
                     n += 1
         if ev_pair is not None:
             ev_pair[0].record(stream)
-        for tab, buf in wl.tables():
+        if multi:
+            # every batch's decode kernel as one chain, then the combines
+            K.paged_decode_attn_multi(wl.pool.handle, [buf.batch() for _, buf in wl.tables()], stream)
+            n += 2 * len(wl.tables())
+        for tab, buf in (() if multi else wl.tables()):
             if fuse_sync and tab is not None:
                 # table sync, append and attention: the decode launch carries
                 # the sync when it fits (else a sync kernel runs first; those
@@ -583,6 +592,7 @@ def main():
               "pool": args.pool if args.workload == "llama8b" else "fixed",
               "append": "separate kernel" if args.separate_append else "fused into attention",
               "table_sync": ("carried by the decode launch when it fits" if fuse_sync else "separate kernel"),
+              "batches": "one paged_decode_attn_multi call" if multi else "one call per batch",
               "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
                                 else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,
               "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}

@@ -525,6 +525,37 @@ int paged_decode_attn_seqtab(kv_pool *pool, kv_seqtab *t, const uint16_t *q, con
                              void *stream);
 
 /*
+ * Several decode batches in one call: co-located models, each with its own
+ * layout, queries, tables and workspace, attending over the one pool.  The
+ * result is that of calling paged_decode_attn (k_new / v_new NULL) or
+ * paged_decode_attn_append for batches[0], batches[1], ... in order, with
+ * num_splits = 0.  The decode kernels run as a chain: each later batch's
+ * kernel starts on the SMs the one before frees as its last warps finish,
+ * and the split-K merges of all batches follow.  Batches must not share a
+ * workspace or an output, and no batch may read a block that another one
+ * appends to (blocks of different layouts never overlap).  All arguments
+ * are checked before anything is launched; errors are those of
+ * paged_decode_attn.  Batches with S = 0 are skipped.
+ */
+typedef struct kv_attn_batch {
+    int layout;
+    const uint16_t *q;      /* [S][Hq][d] */
+    const uint16_t *k_new;  /* [S][Hkv][d] or NULL (no append) */
+    const uint16_t *v_new;  /* [S][Hkv][d] or NULL */
+    uint16_t *out;          /* [S][Hq][d] */
+    const int32_t *dev_table;
+    const int32_t *dev_ctx_lens;
+    int max_blocks;
+    int S;
+    int Hq;
+    float scale;
+    void *workspace;        /* kv_workspace_bytes(pool, layout, S, Hq, max_blocks, 0) */
+    size_t ws_bytes;
+} kv_attn_batch;
+
+int paged_decode_attn_multi(kv_pool *pool, int n, const kv_attn_batch *batches, void *stream);
+
+/*
  * Shared-prefix ("cascade") decode attention.  Sequences that hold the same
  * physical blocks at the start of their block tables -- a system prompt
  * shared by reference by every stage of an agent workflow (§III-B, §III-C)

@@ -98,6 +98,11 @@ struct AttnArgs {
     const int32_t *skip;
     const float *ws_pre;
     int32_t KS;
+    // place in a chain of grids: 0 alone (release the next grid, then wait
+    // for the one before); 1 first of a chain (wait, then release: the next
+    // grid relies on this wait); 2 chained (release, no wait at the start,
+    // a wait at every exit: see the kernel)
+    int32_t chain;
     // fused table sync (paged_decode_attn_seqtab): this step's lengths of
     // rows [0, sync_nlens) and its changed table entries travel here.  The
     // kernel takes the lengths and those entries from here, and the CTAs
@@ -495,7 +500,7 @@ struct Piece {
 // to the table's reach with the error reported.
 __device__ __forceinline__ int32_t load_len(const AttnArgs &a, int s, int32_t *raw_out)
 {
-    const int32_t raw = a.sync_table ? a.sync_words[s] : ld_prior(a.ctx_lens + s, a.skip != nullptr);
+    const int32_t raw = a.sync_table ? a.sync_words[s] : ld_prior(a.ctx_lens + s, a.chain == 2);
     const int32_t cap = a.max_blocks * a.bs;
     *raw_out = raw;
     if (raw < 0 || raw > cap) {
@@ -563,7 +568,7 @@ __device__ __forceinline__ int32_t table_entry(const AttnArgs &a, int64_t idx)
         for (int j = 0; j < a.sync_npatch; ++j)
             if (pw[2 * j] == idx) return pw[2 * j + 1];
     }
-    return ld_prior(a.table + idx, a.skip != nullptr);
+    return ld_prior(a.table + idx, a.chain == 2);
 }
 
 // Pool row of unit u's K tile (TMA y coordinate; V is Hkv*bs rows further),
@@ -643,17 +648,21 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     }
     if (tid == 32) prefetch_tensormap(&tmap);
     // Launched as a programmatic dependent: everything above touches only
-    // this CTA.  Outside shared-prefix mode, wait here for the grid before
-    // (lengths, table, pool writes).  In shared-prefix mode the grid before
-    // is the prefix kernel, which released this grid only after its own wait
-    // had seen every earlier grid complete (plan, table sync, the previous
-    // step's combine); this grid does not wait for the prefix kernel here,
-    // so the two run side by side on disjoint SMs, and waits for it at its
-    // end (cascade_done), so that the combine after it sees both grids'
-    // records.  Data from earlier grids is then read through L2 (ld_prior).
-    grid_launch_dependents();
-    if (!a.skip) grid_dependency_wait();
-    const bool cascade_done = a.skip != nullptr;
+    // this CTA.  Alone (chain 0), release the next grid and wait here for
+    // the grid before (lengths, table, pool writes).  A chained grid (chain
+    // 2: the decode kernel beside the shared-prefix kernel, or the second
+    // and later batches of paged_decode_attn_multi) follows a grid that
+    // released it only after its own wait had seen every earlier grid
+    // complete; it does not wait for that grid here, so the two run side by
+    // side (the later one's CTAs take the SMs the earlier one frees), and
+    // waits for it at every exit (`chained`), so that a combine after it
+    // sees every chained grid's records.  Data from earlier grids is then
+    // read through L2 (ld_prior).  The first grid of a chain (chain 1)
+    // waits before it releases the next.
+    if (a.chain != 1) grid_launch_dependents();
+    if (a.chain != 2) grid_dependency_wait();
+    if (a.chain == 1) grid_launch_dependents();
+    const bool chained = a.chain == 2;
     if (a.sync_table) {
         // fused table sync: the grids before have completed (the wait
         // above), and no CTA of this grid reads what is written here
@@ -722,7 +731,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     const int64_t NP = np_min < (int64_t)a.P * kWarps ? np_min : (int64_t)a.P * kWarps;
     const int64_t first_part = (int64_t)blockIdx.x * kWarps;
     if (first_part >= NP) {
-        if (cascade_done) grid_dependency_wait();
+        if (chained) grid_dependency_wait();
         return;
     }
     const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
@@ -739,7 +748,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
 
     const int64_t part = first_part + warp;
     if (part >= NP) {  // no CTA-wide barrier below this point
-        if (cascade_done) grid_dependency_wait();
+        if (chained) grid_dependency_wait();
         return;
     }
     const int32_t u0 = (int32_t)(part * W / NP);
@@ -853,7 +862,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             a.ws_run[r] = make_int2(p_first, split ? p_last - p_first + 1 : 0);
         u = pc.pe;
     }
-    if (cascade_done) grid_dependency_wait();
+    if (chained) grid_dependency_wait();
 }
 
 // ------------------------------------------------------------ combine ---

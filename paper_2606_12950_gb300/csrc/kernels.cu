@@ -446,6 +446,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.ws_run = reinterpret_cast<int2 *>(ws);
     a.ws_part = reinterpret_cast<float *>(ws + part_off);
     a.skip = c->ws_skip;
+    a.chain = 2;  // beside the prefix kernel, which waits before releasing it
     a.ws_pre = c->ws_pre;
     a.KS = c->KS;
     rc = ensure_tmap(p, layout);
@@ -503,6 +504,102 @@ int paged_decode_attn_seqtab(kv_pool *p, kv_seqtab *t, const uint16_t *q, const 
     const FusedSync sync{t, dev_table, dev_ctx_lens};
     return attn_call(p, t->layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, t->max_blocks, S, Hq, scale,
                      num_splits, workspace, ws_bytes, stream, nullptr, &sync);
+}
+
+// One launch-ready batch of paged_decode_attn_multi.
+struct MultiItem {
+    kvp::AttnArgs a;
+    int variant, D, G, layout, P;
+};
+
+// paged_decode_attn(_append) arguments of one batch checked and turned into
+// launch parameters; nothing is launched.  S == 0 gives *skip = true.
+int prepare_plain(kv_pool *p, const kv_attn_batch &b, MultiItem *it, bool *skip)
+{
+    int G = 0;
+    *skip = false;
+    if (!std::isfinite(b.scale)) return KV_ERR_INVALID_ARG;
+    int rc = attn_shape(p, b.layout, b.S, b.Hq, b.max_blocks, &G);
+    if (rc) return rc;
+    if (b.S == 0) {
+        *skip = true;
+        return KV_OK;
+    }
+    if (!b.q || !b.out || !b.dev_table || !b.dev_ctx_lens || !aligned16(b.q) || !aligned16(b.out))
+        return KV_ERR_INVALID_ARG;
+    if ((b.k_new || b.v_new) && (!b.k_new || !b.v_new || !aligned16(b.k_new) || !aligned16(b.v_new)))
+        return KV_ERR_INVALID_ARG;
+    if (p->sm_count <= 0) return KV_ERR_CUDA;
+    const kv_layout &L = p->desc.layouts[b.layout];
+    kvp::AttnArgs &a = it->a;
+    a = kvp::AttnArgs{};
+    a.q = b.q;
+    a.out = b.out;
+    a.k_new = b.k_new;
+    a.v_new = b.v_new;
+    a.pool = reinterpret_cast<uint16_t *>(p->desc.device_base);
+    a.table = b.dev_table;
+    a.ctx_lens = b.dev_ctx_lens;
+    a.err = p->desc.device_error;
+    a.rows_per_page = (int64_t)(p->page_bytes / (2ull * L.head_dim));
+    a.pool_pages = p->n_pages;
+    a.pages_per_block = p->pages_per_block[b.layout];
+    a.max_blocks = b.max_blocks;
+    a.S = b.S;
+    a.Hkv = L.num_kv_heads;
+    a.bs = p->desc.block_size;
+    a.qk_scale = b.scale * 1.4426950408889634f;
+    it->variant = pick_variant(p, G);
+    it->D = L.head_dim;
+    it->G = G;
+    it->layout = b.layout;
+    int P = 0;
+    rc = dispatch(it->variant, L.head_dim, G, nullptr, &a, 0, p->sm_count, nullptr, kvp::kLaunchQuery, &P);
+    if (rc) return rc;
+    it->P = P;
+    size_t part_off;
+    const size_t need = ws_layout(b.S, L.num_kv_heads, G, L.head_dim, P, &part_off);
+    if (!b.workspace || b.ws_bytes < need || ((uintptr_t)b.workspace & 255u)) return KV_ERR_WORKSPACE;
+    a.ws_run = reinterpret_cast<int2 *>(b.workspace);
+    a.ws_part = reinterpret_cast<float *>(reinterpret_cast<uint8_t *>(b.workspace) + part_off);
+    return ensure_tmap(p, b.layout);
+}
+
+int paged_decode_attn_multi(kv_pool *p, int n, const kv_attn_batch *batches, void *stream)
+{
+    if (!p || n < 0 || (n > 0 && !batches)) return KV_ERR_INVALID_ARG;
+    // every batch is checked before anything is launched
+    std::vector<MultiItem> items;
+    items.reserve((size_t)n);
+    for (int i = 0; i < n; ++i) {
+        MultiItem it;
+        bool skip = false;
+        int rc = prepare_plain(p, batches[i], &it, &skip);
+        if (rc) return rc;
+        if (!skip) items.push_back(it);
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    int P = 0;
+    if (items.size() == 1) {
+        MultiItem &it = items[0];
+        return dispatch(it.variant, it.D, it.G, &p->tmap[it.layout], &it.a, it.P, p->sm_count, st,
+                        kvp::kLaunchBoth, &P);
+    }
+    // the decode kernels as a chain (each later one starts on the SMs the one
+    // before frees and waits for it at its end), then the combines
+    for (size_t i = 0; i < items.size(); ++i) {
+        MultiItem &it = items[i];
+        it.a.chain = i == 0 ? 1 : 2;
+        int rc = dispatch(it.variant, it.D, it.G, &p->tmap[it.layout], &it.a, it.P, p->sm_count, st,
+                          kvp::kLaunchAttention, &P);
+        if (rc) return rc;
+    }
+    for (MultiItem &it : items) {
+        int rc = dispatch(it.variant, it.D, it.G, &p->tmap[it.layout], &it.a, it.P, p->sm_count, st,
+                          kvp::kLaunchCombine, &P);
+        if (rc) return rc;
+    }
+    return KV_OK;
 }
 
 }  // extern "C"

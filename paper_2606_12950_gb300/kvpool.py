@@ -135,6 +135,14 @@ class kv_prefix_group(ctypes.Structure):
     _fields_ = [("count", ctypes.c_int32), ("tokens", ctypes.c_int32)]
 
 
+class kv_attn_batch(ctypes.Structure):
+    _fields_ = [("layout", ctypes.c_int), ("q", ctypes.c_void_p), ("k_new", ctypes.c_void_p),
+                ("v_new", ctypes.c_void_p), ("out", ctypes.c_void_p), ("dev_table", ctypes.c_void_p),
+                ("dev_ctx_lens", ctypes.c_void_p), ("max_blocks", ctypes.c_int), ("S", ctypes.c_int),
+                ("Hq", ctypes.c_int), ("scale", ctypes.c_float), ("workspace", ctypes.c_void_p),
+                ("ws_bytes", ctypes.c_size_t)]
+
+
 KV_ENGINE_IDLE, KV_ENGINE_SLEEPING, KV_ENGINE_SLEEP_PENDING, KV_ENGINE_ACTIVE, KV_ENGINE_COLD = 0, 1, 2, 3, 4
 KV_ACT_SLEEP, KV_ACT_EVICT, KV_ACT_STOP, KV_ACT_PREEMPT, KV_ACT_ABORT = 1, 2, 3, 4, 5
 
@@ -170,6 +178,7 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn_noalloc": [P, I, P, P, P, P, I, I, I, F, I, P],
             "paged_decode_attn_append": [P, I, P, P, P, P, P, P, I, I, I, F, I, P, SZ, P],
             "paged_decode_attn_seqtab": [P, P, P, P, P, P, P, P, I, I, F, I, P, SZ, P],
+            "paged_decode_attn_multi": [P, I, P, P],
             "kv_set_attn_variant": [P, I],
             "kv_cascade_workspace_bytes": [P, I, I, I, I, ctypes.POINTER(SZ)],
             "kv_pool_create_vmm": [ctypes.POINTER(kv_pool_desc), ctypes.POINTER(kv_vmm_desc), ctypes.POINTER(P)],
@@ -429,6 +438,26 @@ def paged_decode_attn_seqtab(pool, seqtab, q, k_new, v_new, out, dev_table, dev_
            lib().paged_decode_attn_seqtab(pool, h, _addr(q), _addr(k_new), _addr(v_new), _addr(out),
                                           _addr(dev_table), _addr(dev_ctx_lens), int(S), int(Hq), float(scale),
                                           int(num_splits), _addr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def attn_batches(batches) -> "ctypes.Array":
+    """kv_attn_batch array from dicts with the struct's fields (tensors or
+    addresses for the pointers; k_new / v_new None for no append)."""
+    arr = (kv_attn_batch * max(1, len(batches)))()
+    for i, b in enumerate(batches):
+        arr[i] = kv_attn_batch(int(b["layout"]), _addr(b["q"]), _addr(b.get("k_new")), _addr(b.get("v_new")),
+                               _addr(b["out"]), _addr(b["dev_table"]), _addr(b["dev_ctx_lens"]),
+                               int(b["max_blocks"]), int(b["S"]), int(b["Hq"]), float(b["scale"]),
+                               _addr(b["workspace"]), int(b["ws_bytes"]))
+    return arr
+
+
+def paged_decode_attn_multi(pool, batches, stream=None) -> None:
+    """Several batches (co-located layouts) in one call; `batches` is a
+    kv_attn_batch array (attn_batches) or a list of dicts."""
+    arr = batches if isinstance(batches, ctypes.Array) else attn_batches(batches)
+    n = len(batches)
+    _check("paged_decode_attn_multi", lib().paged_decode_attn_multi(pool, n, ctypes.addressof(arr), _stream(stream)))
 
 
 def paged_decode_attn_noalloc(pool, layout: int, q, out, dev_table, dev_ctx_lens, max_blocks: int, S: int,

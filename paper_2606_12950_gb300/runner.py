@@ -188,6 +188,13 @@ class DeviceBatch:
                                    self.table, self.lens, self.max_blocks, self.S, self.Hq, self.b.scale,
                                    self.num_splits, self.ws, self.ws.numel(), stream)
 
+    def batch(self, fused: bool = True) -> dict:
+        """This batch as a paged_decode_attn_multi entry."""
+        return {"layout": self.layout, "q": self.q, "k_new": self.k_new if fused else None,
+                "v_new": self.v_new if fused else None, "out": self.out, "dev_table": self.table,
+                "dev_ctx_lens": self.lens, "max_blocks": self.max_blocks, "S": self.S, "Hq": self.Hq,
+                "scale": self.b.scale, "workspace": self.ws, "ws_bytes": self.ws.numel()}
+
     def cascade(self, plan, fused: bool = True, stream=None) -> None:
         """Shared-prefix attention (with the fused append unless fused=False)."""
         need = K.kv_cascade_workspace_bytes(self.pool.handle, self.layout, self.S, self.Hq, self.max_blocks)
@@ -258,6 +265,13 @@ class DeviceSteps:
         K.paged_decode_attn_append(self.pool.handle, self.layout, self.q, self.k_new, self.v_new, self.out,
                                    self.table, self.lens, self.max_blocks, self.S, self.Hq, self.scale,
                                    self.num_splits, self.ws, self.ws.numel(), stream)
+
+    def batch(self, fused: bool = True) -> dict:
+        """This batch as a paged_decode_attn_multi entry."""
+        return {"layout": self.layout, "q": self.q, "k_new": self.k_new if fused else None,
+                "v_new": self.v_new if fused else None, "out": self.out, "dev_table": self.table,
+                "dev_ctx_lens": self.lens, "max_blocks": self.max_blocks, "S": self.S, "Hq": self.Hq,
+                "scale": self.scale, "workspace": self.ws, "ws_bytes": self.ws.numel()}
 
     def sync_append_attend(self, seqtab, stream=None) -> None:
         """seqtab's table sync, the append and the attention: one launch of

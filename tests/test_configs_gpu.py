@@ -163,6 +163,49 @@ def test_colocated_models_full_size():
     pool.close()
 
 
+def test_colocated_models_in_one_multi_call():
+    """The three co-located batches in one paged_decode_attn_multi call (the
+    decode kernels chained, then the combines), with the fused append:
+    outputs and pool bit-identical to three paged_decode_attn_append calls,
+    and the oracle's values on sampled sequences.  A batch with S = 0 in the
+    list is skipped."""
+    from paper_2606_12950_gb300 import kvpool as K
+    from paper_2606_12950_gb300.runner import DeviceBatch, DevicePool
+
+    batches, n_pages, page_elems = W.config4_colocation()
+    sides = []
+    for _ in range(2):
+        pool = DevicePool(n_pages, page_elems * 2, 16, [(b.Hkv, b.d) for b in batches])
+        pool.upload(batches[0].pool)
+        sides.append((pool, [DeviceBatch(pool, li, b) for li, b in enumerate(batches)]))
+    pool_a, dbs_a = sides[0]
+    for db in dbs_a:
+        db.append_attend()
+    pool_b, dbs_b = sides[1]
+    entries = [db.batch() for db in dbs_b]
+    empty = dict(entries[1], S=0)
+    K.paged_decode_attn_multi(pool_b.handle, [entries[0], empty, entries[1], entries[2]])
+    torch.cuda.synchronize()
+    got_pool = pool_b.download()
+    assert np.array_equal(pool_a.download(), got_pool)
+    for li in range(3):
+        assert np.array_equal(dbs_a[li].out_bits(), dbs_b[li].out_bits()), f"layout {li}"
+    host_pool = batches[0].pool.copy()
+    for b in batches:
+        oracle.append(host_pool, n_pages, page_elems, b.bs, b.Hkv, b.d, b.k_new, b.v_new, b.table, b.ctx_lens,
+                      inplace=True)
+    assert np.array_equal(got_pool, host_pool)
+    rng = np.random.default_rng(12)
+    for li, (b, db) in enumerate(zip(batches, dbs_b)):
+        ids = _sample(rng, b.ctx_lens, 8)
+        ref = oracle.paged_attention(host_pool, n_pages, page_elems, b.bs, b.Hkv, b.d, b.q, b.table, b.ctx_lens,
+                                     b.scale, seq_ids=ids)
+        _check(db.out_f64()[ids], ref[ids], f"layout {li}")
+    assert pool_a.error() == 0 and pool_b.error() == 0
+    for pool, _ in sides:
+        pool.close()
+
+
 def test_long_context_stress_full_size():
     """1024 sequences, bounded-Pareto(1.2) contexts on [256, 131072], bs=32:
     steps with appends, sequences finishing, blocks freed and reused by new
