@@ -57,7 +57,8 @@ constexpr uint32_t kHalfBytes = kTile * 128;      // one 64-column box: 16 rows 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
 // Loads of data written by earlier grids: through L2 only (ld.global.cg) when
-// the kernel did not wait for the grid before it (shared-prefix mode), so that
+// the kernel did not wait for the grid before it (a chained grid: beside the
+// shared-prefix kernel, or a later batch of paged_decode_attn_multi), so that
 // no line an earlier kernel left in this SM's L1 is read; plain otherwise.
 template <class T>
 __device__ __forceinline__ T ld_prior(const T *p, bool l2_only)
