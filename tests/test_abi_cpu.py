@@ -167,3 +167,20 @@ def test_attention_argument_checks_precede_any_launch():
     # S = 0 is a no-op that needs no buffers
     K.paged_decode_attn(h, 0, 0, 0, 0, 0, 8, 0, 32, 0.1, 0, 0, 0)
     K.kv_append(h, 0, 0, 0, 0, 0, 8, 0)
+
+
+def test_multi_batch_checks_every_batch_before_launching():
+    h, _ = make_pool(n_pages=16)
+    empty = dict(layout=0, q=0, out=0, dev_table=0, dev_ctx_lens=0, max_blocks=8, S=0, Hq=32, scale=0.1,
+                 workspace=0, ws_bytes=0)
+    K.paged_decode_attn_multi(h, [])               # nothing to do
+    K.paged_decode_attn_multi(h, [empty, empty])   # S = 0 batches are skipped: nothing is launched
+    for bad, code in [(dict(empty, S=4, Hq=12), K.KV_ERR_INVALID_ARG),   # Hq not a multiple of Hkv
+                      (dict(empty, S=4, Hq=24), K.KV_ERR_UNSUPPORTED),   # G = 3 is not built
+                      (dict(empty, S=4), K.KV_ERR_INVALID_ARG),          # no q / out / table
+                      (dict(empty, layout=1), K.KV_ERR_INVALID_ARG),     # no layout 1
+                      (dict(empty, scale=float("nan")), K.KV_ERR_INVALID_ARG)]:
+        with pytest.raises(K.KVError) as e:  # a bad batch after a good one: the call launches nothing
+            K.paged_decode_attn_multi(h, [empty, bad])
+        assert e.value.code == code, bad
+    assert K.lib().paged_decode_attn_multi(h, -1, None, None) == K.KV_ERR_INVALID_ARG
