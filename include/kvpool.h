@@ -467,9 +467,10 @@ int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream);
  *     out[s][h] = sum_{j<n} softmax_j(scale * q[s][h] . K_j) V_j
  * with K_j, V_j the rows of head g at position j, found through dev_table.
  * q, out: bf16 [S][Hq][d] arrays, 16-byte aligned, in device memory or in
- * pinned (page-locked, mapped) host memory: the kernels read q and write
- * out with ordinary loads and stores, which on GB300 cross the coherent
- * NVLink-C2C link to host memory, so a caller holding a step's inputs and
+ * pinned (page-locked, mapped) host memory: the kernels read q with
+ * 16-byte copies into shared memory (cp.async) and write out with ordinary
+ * stores, which on GB300 cross the coherent NVLink-C2C link to host
+ * memory, so a caller holding a step's inputs and
  * results on the host needs no separate copies (the same holds for k_new
  * and v_new of the calls below).  The pool, table, lengths and workspace
  * are device memory.  A sequence with n == 0 gets zeros.
