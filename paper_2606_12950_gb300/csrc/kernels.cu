@@ -1,5 +1,9 @@
-// kernels.cu -- KV append kernel and the launch wrappers of the C ABI
-// (kv_append, kv_workspace_bytes, paged_decode_attn).
+// kernels.cu -- KV append kernel, the shared-prefix plan kernel and the
+// launch wrappers of the C ABI: kv_append, kv_workspace_bytes,
+// kv_cascade_workspace_bytes, paged_decode_attn(_append), the table sync
+// carried by the decode launch (paged_decode_attn_seqtab), co-located
+// batches as one chain (paged_decode_attn_multi) and shared-prefix
+// attention (paged_decode_attn_cascade).
 #include <algorithm>
 #include <cmath>
 #include <memory>
@@ -193,7 +197,8 @@ size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
 }
 
 // cascade workspace: the above, then the per-sequence skip (padded to 256
-// bytes), then kMaxKeySplits prefix records per (sequence, KV head)
+// bytes), the plan words (kCascadeWords, padded), then kMaxKeySplits prefix
+// records per (sequence, KV head)
 size_t cascade_ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off, size_t *skip_off, size_t *pre_off,
                          size_t *plan_off)
 {
