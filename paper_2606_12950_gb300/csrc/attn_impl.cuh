@@ -26,9 +26,18 @@
 // next q.K.  (Measured on GB300: one issuing thread per SM cannot keep HBM
 // busy with these 2 KB boxes; one per warp can.)  The pool rows of the CTA's
 // units are resolved from the block table in the prologue, while the memory
-// system is idle, so no table load sits on the streaming path.  A run that
-// ends inside a warp's range is written out by that warp directly; no state
-// is merged between warps of a CTA.
+// system is idle, so no table load sits on the streaming path, and each
+// run's q rows (and, for the run's last tile, this step's new K/V rows) are
+// staged into the warp's shared buffers by cp.async one piece ahead.  A run
+// that ends inside a warp's range is written out by that warp directly; no
+// state is merged between warps of a CTA.
+//
+// Grid-to-grid order: the kernel is launched as a programmatic dependent.
+// Alone it releases the next grid and waits for the one before; as part of
+// a chain (beside the shared-prefix kernel, or the later batches of several
+// co-located ones) it starts without waiting, reads what earlier grids wrote
+// through L2 only, and waits at its end (AttnArgs::chain).  The step's
+// table sync may ride in its parameters (AttnArgs::sync_words).
 //
 // Two compute variants share this skeleton:
 //   FmaCompute : CUDA-core FFMA2 dot products and weighted sums.
