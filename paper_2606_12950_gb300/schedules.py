@@ -116,8 +116,7 @@ class LongContextStress:
             self._admit(s)
 
     def _admit(self, s: int) -> bool:
-        n = int(W.config5_lengths(self.rng, 1)[0])
-        budget = int(W.config5_budgets(self.rng, 1)[0])
+        n, budget = W.config5_draw(self.rng)
         try:
             self.tab.reserve(s, n + budget)  # the whole run, Eq. 2 with the true length
         except K.KVError as e:
