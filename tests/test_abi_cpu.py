@@ -184,3 +184,24 @@ def test_multi_batch_checks_every_batch_before_launching():
             K.paged_decode_attn_multi(h, [empty, bad])
         assert e.value.code == code, bad
     assert K.lib().paged_decode_attn_multi(h, -1, None, None) == K.KV_ERR_INVALID_ARG
+
+
+def test_seqtab_attention_argument_checks_precede_any_launch():
+    h, _ = make_pool(n_pages=16)
+    h2, _ = make_pool(n_pages=16)
+    t = K.SeqTab(h, 0, 4, 8)
+    fake = 1 << 41  # never dereferenced: every call below fails its host checks
+    cases = [
+        (h2, t, dict(S=4), K.KV_ERR_INVALID_ARG),                  # table over another pool
+        (h, t, dict(S=5), K.KV_ERR_INVALID_ARG),                   # more rows than the table has
+        (h, t, dict(S=4, dev_table=None), K.KV_ERR_INVALID_ARG),   # no device table
+        (h, t, dict(S=4, v_new=None), K.KV_ERR_INVALID_ARG),       # k_new without v_new
+    ]
+    for pool, tab, over, code in cases:
+        args = dict(q=fake, k_new=fake, v_new=fake, out=fake, dev_table=fake, dev_lens=fake, S=4)
+        args.update(over)
+        with pytest.raises(K.KVError) as e:
+            K.paged_decode_attn_seqtab(pool, tab, args["q"], args["k_new"], args["v_new"], args["out"],
+                                       args["dev_table"], args["dev_lens"], args["S"], 32, 0.1, 0, fake, 1 << 20)
+        assert e.value.code == code, over
+    t.close()
