@@ -498,12 +498,6 @@ def main():
     time.sleep(0.3)
     for i in range(args.warmup):
         step()
-    # the attention call is timed with an event pair on every SAMPLE-th step
-    # only: an event between two kernels ends their programmatic overlap, so
-    # pairs on every step would slow the step they are meant to measure
-    SAMPLE = 10
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range((args.steps + SAMPLE - 1) // SAMPLE)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
@@ -514,22 +508,45 @@ def main():
     h0 = time.perf_counter()
     t_start.record(stream)
     for i in range(args.steps):
-        step_bytes.append(step(evs[i // SAMPLE] if i % SAMPLE == 0 else None))
+        step_bytes.append(step())
     t_end.record(stream)
     host_us = (time.perf_counter() - h0) * 1e6 / args.steps  # host submission time per step
     extra_sync_launches = sync_kernels() - sync0 if fuse_sync else 0
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
-    attn_ms = [a.elapsed_time(z) for a, z in evs]
     err = wl.pool.error(stream)
 
     dram_rank = sum(x[0] for x in step_bytes)
     logical_rank = sum(x[1] for x in step_bytes)
-    attn_avg_ms = float(np.mean(attn_ms))
-    sampled = [step_bytes[i][0] for i in range(0, args.steps, SAMPLE)]
-    attn_gbs = float(np.mean(sampled)) / (attn_avg_ms * 1e-3) / 1e9  # this rank's kernels
+    # Every launch in the timed region is one of the attention call's kernels
+    # (the host steps launch nothing), so the region's device time per step
+    # is the call's average duration when the host keeps ahead of the GPU,
+    # and an upper bound on it otherwise: this rank's roofline figure.
+    call_ms = ms / args.steps
+    attn_gbs = dram_rank / args.steps / (call_ms * 1e-3) / 1e9
+    # A second, conservative reading after the timed region: single calls,
+    # each between two events.  An event between two kernels ends their
+    # programmatic overlap, so an isolated call is slower than one inside the
+    # chain of steps.
+    iso = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+    iso_bytes = [step(pair)[0] for pair in iso]
+    torch.cuda.synchronize()
+    iso_ms = float(np.mean([a.elapsed_time(z) for a, z in iso]))
+    iso_gbs = float(np.mean(iso_bytes)) / (iso_ms * 1e-3) / 1e9
     peak, peak_kind = load_peaks()
+    if cascade is not None:
+        step_kernels = ("seqtab_sync_kernel, cascade_plan_kernel, paged_attn_kernel (suffixes, fused append) "
+                        "beside cascade_prefix_kernel, combine_kernel")
+    elif args.separate_append:
+        step_kernels = "seqtab_sync_kernel, append_kernel, paged_attn_kernel, combine_kernel"
+    elif multi:
+        step_kernels = "paged_attn_kernel per batch (fused append, one chain), then combine_kernel per batch"
+    elif fuse_sync:
+        step_kernels = "paged_attn_kernel (fused append and table sync), combine_kernel"
+    else:
+        step_kernels = (("seqtab_sync_kernel, " if any(t is not None for t, _ in wl.tables()) else "")
+                        + "paged_attn_kernel (fused append), combine_kernel")
 
     # end to end: each step's q / k / v come from pinned host memory and its
     # output goes back to pinned host memory.  The C-ABI calls get the host
@@ -603,10 +620,12 @@ def main():
         "decode_tokens_per_s": tokens_per_s,
         "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peak, "unit": "GB/s",
                      "frac": attn_gbs / peak, "traffic": traffic,
-                     "kernel": "paged_attn_kernel (+ combine_kernel, fused append)",
-                     "peak_kind": peak_kind, "attn_ms": attn_avg_ms,
-                     "timed_launches": len(attn_ms), "timing": f"CUDA events around every {SAMPLE}th step's "
-                                                                 "attention call in the timed region"},
+                     "kernel": step_kernels,
+                     "peak_kind": peak_kind, "call_ms": call_ms, "timed_launches": launches_per_step * args.steps
+                     + extra_sync_launches,
+                     "timing": "CUDA events at the ends of the timed region, whose launches are all the "
+                               "attention call's kernels: region time / steps",
+                     "isolated_call_ms": iso_ms, "isolated_frac": iso_gbs / peak},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps + extra_sync_launches,

@@ -306,6 +306,26 @@ int kv_seq_release(kv_seqtab *t, int s);
 int kv_seq_trim(kv_seqtab *t, int s);
 
 /*
+ * A step's finished sequences replaced by new admissions, in one call: for
+ * i = 0 .. n-1 in order, slot slots[i] drops every block reference it holds
+ * (kv_seq_release), then reserves ceil(reserve_tokens[i] / bs) blocks for
+ * the new sequence's whole run (Eq. 2) and takes length lens[i]
+ * (kv_seq_reserve, kv_seq_set_len).  The release of one slot precedes the
+ * next slot's reservation, so freed blocks serve later admissions.
+ *   slots          host int32[n], distinct, each in [0, max_seqs)
+ *   reserve_tokens host int64[n], 0 .. max_blocks * bs
+ *   lens           host int32[n], 0 .. reserve_tokens[i]
+ *   status         host int32[n] out: KV_OK, or KV_ERR_OUT_OF_BLOCKS where the
+ *                  pool could not serve that reservation (the slot is then
+ *                  left empty, length 0, and the admission is the caller's to
+ *                  retry); the call itself still returns KV_OK
+ * Every argument is checked before any slot changes: KV_ERR_INVALID_ARG and
+ * nothing changed.  n = 0 is a no-op.
+ */
+int kv_seq_replace(kv_seqtab *t, int n, const int32_t *slots, const int64_t *reserve_tokens,
+                   const int32_t *lens, int32_t *status);
+
+/*
  * Bring a device copy of the table up to date on `stream`: every slot's
  * length goes to dev_ctx_lens[0 .. max_seqs), and every table entry changed
  * since the previous sync (of this table, to any device copy) goes to

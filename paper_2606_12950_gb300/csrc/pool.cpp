@@ -106,6 +106,7 @@ int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool)
     p->super_free.assign(order.rbegin(), order.rend());
     p->refcnt.assign((size_t)p->n_pages, 0);
     p->owner.assign((size_t)p->n_pages, (int8_t)-1);
+    p->tally.assign((size_t)p->n_pages, 0);
     if (cudaGetDevice(&p->device) != cudaSuccess ||
         cudaDeviceGetAttribute(&p->sm_count, cudaDevAttrMultiProcessorCount, p->device) != cudaSuccess) {
         // host-only use (no GPU visible): allocation still works; launches will fail
@@ -162,19 +163,24 @@ int kv_alloc_blocks(kv_pool *p, int layout, int n, int32_t *out_ids)
 
 static int check_live(kv_pool *p, int layout, int n, const int32_t *ids, bool for_free)
 {
-    std::unordered_map<int32_t, int32_t> seen;
-    for (int i = 0; i < n; ++i) {
+    // a free may name an id at most refcnt times: counted in the pool's
+    // per-page tally, which is back to all zeros when the check returns
+    int rc = KV_OK;
+    int i = 0;
+    for (; i < n; ++i) {
         int32_t id = ids[i];
-        if (id < 0 || id >= p->n_pages) return KV_ERR_INVALID_ARG;
-        if (p->owner[(size_t)id] != layout || p->refcnt[(size_t)id] <= 0) return KV_ERR_INVALID_ARG;
+        if (id < 0 || id >= p->n_pages) { rc = KV_ERR_INVALID_ARG; break; }
+        if (p->owner[(size_t)id] != layout || p->refcnt[(size_t)id] <= 0) { rc = KV_ERR_INVALID_ARG; break; }
         if (for_free) {
-            int32_t c = ++seen[id];
-            if (c > p->refcnt[(size_t)id]) return KV_ERR_INVALID_ARG;
+            if (++p->tally[(size_t)id] > p->refcnt[(size_t)id]) { rc = KV_ERR_INVALID_ARG; ++i; break; }
         } else if (p->refcnt[(size_t)id] == INT32_MAX) {
-            return KV_ERR_INVALID_ARG;
+            rc = KV_ERR_INVALID_ARG;
+            break;
         }
     }
-    return KV_OK;
+    if (for_free)
+        for (int j = 0; j < i; ++j) p->tally[(size_t)ids[j]] = 0;
+    return rc;
 }
 
 int kv_free_blocks(kv_pool *p, int layout, int n, const int32_t *ids)

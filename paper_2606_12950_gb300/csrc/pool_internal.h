@@ -43,6 +43,7 @@ struct kv_pool {
     std::vector<int32_t> free_blocks[KV_MAX_LAYOUTS];  // LIFO stacks of block ids
     std::vector<int32_t> refcnt;              // per page id (block start); 0 = not live
     std::vector<int8_t> owner;                // layout owning the block at page id, -1 none
+    std::vector<int32_t> tally;               // per page id, all 0 between calls: duplicate counts of a free
     int64_t used_blocks[KV_MAX_LAYOUTS];
     int64_t carved_blocks[KV_MAX_LAYOUTS];    // blocks cut from superpages so far
     int device = 0;

@@ -102,10 +102,11 @@ int kv_seq_reserve(kv_seqtab *t, int s, int64_t tokens)
     const int h = t->held[(size_t)s];
     if (need <= h) return KV_OK;
     const int n = (int)(need - h);
-    std::vector<int32_t> ids((size_t)n);
-    int rc = kv_alloc_blocks(t->pool, t->layout, n, ids.data());
-    if (rc) return rc;
-    for (int k = 0; k < n; ++k) set_entry(t, s, h + k, ids[(size_t)k]);
+    // the new ids land in the row's free tail (all -1), then are marked changed
+    int32_t *row = &t->table[(size_t)s * t->max_blocks];
+    int rc = kv_alloc_blocks(t->pool, t->layout, n, row + h);
+    if (rc) return rc;  // nothing written
+    for (int k = 0; k < n; ++k) set_entry(t, s, h + k, row[h + k]);
     t->held[(size_t)s] = (int32_t)need;
     t->counters.blocks_held += n;
     return KV_OK;
@@ -185,6 +186,38 @@ int kv_seq_trim(kv_seqtab *t, int s)
     for (int i = keep; i < h; ++i) set_entry(t, s, i, -1);
     t->held[(size_t)s] = keep;
     t->counters.blocks_held -= h - keep;
+    return KV_OK;
+}
+
+int kv_seq_replace(kv_seqtab *t, int n, const int32_t *slots, const int64_t *reserve_tokens,
+                   const int32_t *lens, int32_t *status)
+{
+    if (!t || !t->pool || n < 0) return KV_ERR_INVALID_ARG;
+    if (n == 0) return KV_OK;
+    if (!slots || !reserve_tokens || !lens || !status) return KV_ERR_INVALID_ARG;
+    const int64_t cap = (int64_t)t->max_blocks * t->bs;
+    std::vector<uint8_t> seen((size_t)t->S, 0);
+    for (int i = 0; i < n; ++i) {
+        const int32_t s = slots[i];
+        if (!slot_ok(t, s) || seen[(size_t)s]) return KV_ERR_INVALID_ARG;
+        seen[(size_t)s] = 1;
+        if (reserve_tokens[i] < 0 || reserve_tokens[i] > cap) return KV_ERR_INVALID_ARG;
+        if (lens[i] < 0 || (int64_t)lens[i] > reserve_tokens[i]) return KV_ERR_INVALID_ARG;
+    }
+    for (int i = 0; i < n; ++i) {
+        const int32_t s = slots[i];
+        int rc = KV_OK;
+        if (t->held[(size_t)s] > 0 || t->lens[(size_t)s] > 0) rc = kv_seq_release(t, s);
+        if (rc) return rc;
+        rc = kv_seq_reserve(t, s, reserve_tokens[i]);
+        if (rc == KV_ERR_OUT_OF_BLOCKS) {
+            status[i] = rc;  // the slot stays empty
+            continue;
+        }
+        if (rc) return rc;
+        t->lens[(size_t)s] = lens[i];
+        status[i] = KV_OK;
+    }
     return KV_OK;
 }
 

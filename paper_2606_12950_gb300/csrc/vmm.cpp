@@ -295,6 +295,7 @@ int kv_pool_create_vmm(const kv_pool_desc *desc, const kv_vmm_desc *vmm, kv_pool
     p->n_pages = n_chunks * spc * p->super_pages;
     p->refcnt.assign((size_t)p->n_pages, 0);
     p->owner.assign((size_t)p->n_pages, (int8_t)-1);
+    p->tally.assign((size_t)p->n_pages, 0);
     p->super_free.clear();
     kv_vmm_state &v = p->vmm;
     v.active = true;

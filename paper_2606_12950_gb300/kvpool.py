@@ -196,6 +196,7 @@ def lib() -> ctypes.CDLL:
             "kv_seq_advance": [P, I, P, ctypes.POINTER(I32)],
             "kv_seq_release": [P, I],
             "kv_seq_trim": [P, I],
+            "kv_seq_replace": [P, I, P, P, P, P],
             "kv_seqtab_sync": [P, P, P, P],
             "kv_seqtab_host": [P, ctypes.POINTER(P), ctypes.POINTER(P)],
             "kv_seqtab_get_counters": [P, ctypes.POINTER(kv_seqtab_counters)],
@@ -519,9 +520,11 @@ class SeqTab:
         self.handle = h.value
         self.S = int(max_seqs)
         self.max_blocks = int(max_blocks)
+        self._lens_view = None
 
     def close(self) -> None:
         if self.handle:
+            self._lens_view = None
             _check("kv_seqtab_destroy", lib().kv_seqtab_destroy(self.handle))
             self.handle = None
 
@@ -549,6 +552,21 @@ class SeqTab:
     def trim(self, s: int) -> None:
         _check("kv_seq_trim", lib().kv_seq_trim(self.handle, int(s)))
 
+    def replace(self, slots, reserve_tokens, lens) -> np.ndarray:
+        """Release each listed slot, then reserve and set the length of its
+        new sequence, in order (kv_seq_replace).  Returns the per-slot status:
+        0, or KV_ERR_OUT_OF_BLOCKS where that admission found the pool full
+        (the slot is left empty)."""
+        a = _i32(slots)
+        r = np.ascontiguousarray(reserve_tokens, dtype=np.int64)
+        n = _i32(lens)
+        if not (a.shape == r.shape == n.shape and a.ndim == 1):
+            raise ValueError("slots, reserve_tokens and lens must be 1-D and of one length")
+        st = np.zeros(a.size, dtype=np.int32)
+        _check("kv_seq_replace", lib().kv_seq_replace(self.handle, int(a.size), a.ctypes.data, r.ctypes.data,
+                                                      n.ctypes.data, st.ctypes.data))
+        return st
+
     def sync(self, dev_table, dev_ctx_lens, stream=None) -> None:
         _check("kv_seqtab_sync", lib().kv_seqtab_sync(self.handle, _addr(dev_table), _addr(dev_ctx_lens),
                                                       _stream(stream)))
@@ -564,10 +582,16 @@ class SeqTab:
 
     def lens(self) -> np.ndarray:
         """Copy of the host lengths only."""
-        t = ctypes.c_void_p()
-        l = ctypes.c_void_p()
-        _check("kv_seqtab_host", lib().kv_seqtab_host(self.handle, ctypes.byref(t), ctypes.byref(l)))
-        return np.ctypeslib.as_array(ctypes.cast(l, ctypes.POINTER(ctypes.c_int32)), shape=(self.S,)).copy()
+        if self.handle is None:
+            raise KVError("kv_seqtab_host", KV_ERR_INVALID_ARG)
+        if self._lens_view is None:
+            # the table's length array keeps its address for the table's life;
+            # the view is dropped when the table closes
+            t = ctypes.c_void_p()
+            l = ctypes.c_void_p()
+            _check("kv_seqtab_host", lib().kv_seqtab_host(self.handle, ctypes.byref(t), ctypes.byref(l)))
+            self._lens_view = np.ctypeslib.as_array(ctypes.cast(l, ctypes.POINTER(ctypes.c_int32)), shape=(self.S,))
+        return self._lens_view.copy()
 
     def counters(self) -> dict:
         c = kv_seqtab_counters()

@@ -112,32 +112,31 @@ class LongContextStress:
         self.admitted = 0
         self.released = 0
         self.deferred = 0
-        for s in range(S):
-            self._admit(s)
+        self._admit(np.arange(S))
 
-    def _admit(self, s: int) -> bool:
-        n, budget = W.config5_draw(self.rng)
-        try:
-            self.tab.reserve(s, n + budget)  # the whole run, Eq. 2 with the true length
-        except K.KVError as e:
-            if e.code != K.KV_ERR_OUT_OF_BLOCKS:
-                raise
-            self.deferred += 1  # the pool is full: the admission waits (the stage is rejected for now)
-            return False
-        self.tab.set_len(s, n)
-        self.left[s] = budget
-        self.admitted += 1
-        return True
+    def _admit(self, slots: np.ndarray) -> None:
+        """Release the listed slots and admit a new sequence into each, in
+        one library call: a cached length and a decode budget drawn per slot,
+        and a reservation for the whole run (Eq. 2 with the true length).
+        Where the pool is full the admission waits (the slot stays empty and
+        is retried on the next step)."""
+        k = int(slots.size)
+        n = W.config5_lengths(self.rng, k)
+        budget = W.config5_budgets(self.rng, k)
+        status = self.tab.replace(slots, n + budget, n)
+        ok = status == 0
+        self.left[slots[ok]] = budget[ok]
+        self.admitted += int(ok.sum())
+        self.deferred += k - int(ok.sum())
 
     def step(self) -> None:
         lens = self.tab.lens()
-        for s in np.nonzero(self.left == 0)[0]:
-            s = int(s)
-            if lens[s] > 0:
-                self.tab.release(s)
-                self.released += 1
-            self._admit(s)
-        live = np.nonzero(self.tab.lens() > 0)[0].astype(np.int32)
+        done = np.nonzero(self.left == 0)[0]
+        if done.size:
+            self.released += int((lens[done] > 0).sum())
+            self._admit(done)
+            lens = self.tab.lens()
+        live = np.nonzero(lens > 0)[0].astype(np.int32)
         self.tab.advance(live)
         self.left[live] -= 1
 

@@ -349,13 +349,3 @@ def config5_lengths(rng, n: int) -> np.ndarray:
 def config5_budgets(rng, n: int, lo: int = 1, hi: int = 64) -> np.ndarray:
     """decode steps each sequence has left before it finishes (uniform)"""
     return rng.integers(lo, hi + 1, size=n)
-
-
-def config5_draw(rng) -> tuple:
-    """One admission's (cached length, decode budget): the values, and the
-    generator state afterwards, of config5_lengths(rng, 1) followed by
-    config5_budgets(rng, 1), without the per-call cost of one-element arrays
-    (the long-context schedule admits tens of sequences a step)."""
-    u = rng.random()
-    x = 256 / (1.0 - u * (1.0 - (256 / 131072) ** 1.2)) ** (1.0 / 1.2)
-    return min(max(math.floor(x), 256), 131072), int(rng.integers(1, 65))

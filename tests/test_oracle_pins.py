@@ -260,13 +260,3 @@ def test_generator_is_seeded_and_shaped():
     used = a.table[a.table >= 0]
     assert len(set(used.tolist())) == used.size  # no block used twice
     assert used.max() < 128
-
-
-def test_config5_scalar_draw_equals_the_array_draws():
-    """The long-context schedule's one-admission draw gives the same lengths,
-    budgets and generator state as the array functions it stands for."""
-    r1, r2 = np.random.default_rng(11), np.random.default_rng(11)
-    for _ in range(20000):
-        a = (int(W.config5_lengths(r1, 1)[0]), int(W.config5_budgets(r1, 1)[0]))
-        assert W.config5_draw(r2) == a
-    assert r1.random() == r2.random()

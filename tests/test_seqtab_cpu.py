@@ -145,3 +145,87 @@ def test_destroying_the_pool_first_detaches_its_tables():
     t.close()
     assert K.kv_pool_stats(pool)["blocks_used"][0] == 0
     K.kv_pool_destroy(pool)
+
+
+def test_replace_equals_release_reserve_set_len_in_order():
+    """kv_seq_replace against the same operations one call at a time on a
+    twin pool: identical tables (block ids included), lengths and refcounts,
+    and the slot model agrees; a reservation the pool cannot serve leaves
+    its slot empty while later, smaller ones are still admitted."""
+    pool_a, a = make(n_pages=120)
+    pool_b, b = make(n_pages=120)
+    m = SeqModel(12, 40, BS)
+    rng = np.random.default_rng(8)
+    misses = 0
+    for step in range(60):
+        k = int(rng.integers(0, 7))
+        slots = rng.choice(12, k, replace=False).astype(np.int32)
+        res = rng.integers(0, 40 * BS + 1, size=k)
+        res[rng.random(k) < 0.5] //= 8  # many small requests beside the large ones
+        lens = (res * rng.random(k)).astype(np.int32)
+        status = a.replace(slots, res, lens)
+        for i, s in enumerate(slots):
+            s = int(s)
+            b.release(s)
+            m.release(s)
+            try:
+                b.reserve(s, int(res[i]))
+            except K.KVError as e:
+                assert e.code == K.KV_ERR_OUT_OF_BLOCKS
+                assert status[i] == K.KV_ERR_OUT_OF_BLOCKS
+                misses += 1
+                continue
+            assert status[i] == 0
+            b.set_len(s, int(lens[i]))
+            m.reserve(s, int(res[i]))
+            m.set_len(s, int(lens[i]))
+        ta, la = a.host()
+        tb, lb = b.host()
+        assert np.array_equal(ta, tb) and np.array_equal(la, lb), step
+        check_rows(a, m, pool_a)
+        live = [s for s in range(12) if m.len[s] > 0 and m.len[s] + 1 <= m.held[s] * BS]
+        if live:
+            a.advance(live)
+            b.advance(live)
+            for s in live:
+                m.len[s] += 1
+    assert misses > 0  # the full-pool branch was taken
+    a.close()
+    b.close()
+
+
+def test_replace_reports_a_full_pool_per_slot():
+    pool, t = make(n_pages=8)  # 8 blocks of 16 tokens
+    st = t.replace([0, 1, 2], [5 * BS, 5 * BS, 3 * BS], [10, 10, 3 * BS])
+    assert list(st) == [0, K.KV_ERR_OUT_OF_BLOCKS, 0]
+    _, lens = t.host()
+    assert list(lens[:3]) == [10, 0, 3 * BS]
+    # slot 0 replaced: its 5 blocks come back first, so slot 1's 5 now fit
+    st = t.replace([0, 1], [0, 5 * BS], [0, 1])
+    assert list(st) == [0, 0]
+    assert K.kv_pool_stats(pool)["blocks_used"][0] == 8
+    t.close()
+
+
+def test_replace_checks_every_argument_before_changing_anything():
+    pool, t = make()
+    t.replace([0, 1], [64, 64], [10, 20])
+    before = t.host()
+    used = K.kv_pool_stats(pool)["blocks_used"][0]
+    bad = [
+        ([0, 0], [16, 16], [1, 1]),            # a slot twice
+        ([0, 12], [16, 16], [1, 1]),           # slot out of range
+        ([0, 1], [16, 41 * BS], [1, 1]),       # more than max_blocks
+        ([0, 1], [16, -1], [1, 0]),            # negative reservation
+        ([0, 1], [16, 16], [1, 17]),           # length beyond the reservation
+        ([0, 1], [16, 16], [1, -1]),           # negative length
+    ]
+    for slots, res, lens in bad:
+        with pytest.raises(K.KVError) as e:
+            t.replace(slots, res, lens)
+        assert e.value.code == K.KV_ERR_INVALID_ARG, (slots, res, lens)
+        after = t.host()
+        assert np.array_equal(before[0], after[0]) and np.array_equal(before[1], after[1])
+        assert K.kv_pool_stats(pool)["blocks_used"][0] == used
+    assert len(t.replace([], [], [])) == 0
+    t.close()
