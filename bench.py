@@ -171,6 +171,71 @@ def oracle_baseline(b, budget_s: float):
             return done_bytes / el / 1e9, steps, el
 
 
+def oracle_baseline_parallel(b, budget_s: float, cores):
+    """The same whole decode steps as oracle_baseline, with each step's
+    attention spread over one thread per core: thread i computes the
+    sequences at ranks i, i + T, ... of a longest-first order (the oracle's
+    own seq_ids subset; ctypes releases the interpreter lock during the C
+    call, so the threads run at once).  The append writes the pool in place
+    (the oracle's inplace option) instead of into a fresh copy of it; the
+    oracle's arithmetic is unchanged.  Returns (GB/s, steps, seconds,
+    threads)."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    import oracle
+
+    oracle.build()
+    T = max(1, len(cores))
+    order = np.argsort(-b.ctx_lens.astype(np.int64), kind="stable")
+    subsets = [order[i::T].astype(np.int32) for i in range(T)]
+    pool = np.array(b.pool, dtype=np.uint16, copy=True)  # appended in place below
+    lens = b.ctx_lens.copy()
+    try:
+        before = os.sched_getaffinity(0)
+        os.sched_setaffinity(0, cores)  # threads created below inherit every core
+    except (AttributeError, OSError):
+        before = None
+    try:
+        with ThreadPoolExecutor(T) as ex:
+            t0 = time.perf_counter()
+            done_bytes = 0
+            steps = 0
+            while True:
+                q, kn, vn = W_step_rows(b, steps)
+                oracle.append(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens, inplace=True)
+                outs = list(ex.map(lambda ids: oracle.paged_attention(pool, b.n_pages, b.page_elems, b.bs, b.Hkv,
+                                                                      b.d, q, b.table, lens, b.scale, seq_ids=ids),
+                                   subsets))
+                kv = int(lens.astype(np.int64).sum()) * 2 * b.Hkv * b.d * 2
+                done_bytes += kv + 2 * b.S * b.Hq * b.d * 2 + 2 * b.S * b.Hkv * b.d * 2
+                steps += 1
+                lens = lens + 1
+                el = time.perf_counter() - t0
+                if el >= budget_s or steps >= 1000:
+                    break
+    finally:
+        if before is not None:
+            os.sched_setaffinity(0, before)
+    # every sequence was computed by exactly one thread in the last step
+    covered = sum((~np.isnan(o[:, 0, 0])).astype(np.int64) for o in outs)
+    if not np.all(covered == 1):
+        raise RuntimeError("threaded oracle baseline: the subsets do not cover the batch once")
+    return done_bytes / el / 1e9, steps, el, T
+
+
+def cpu_model() -> str:
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu part", "hardware")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+
+    return platform.processor() or platform.machine()
+
+
 def W_step_rows(b, step):
     from paper_2606_12950_gb300 import workloads as W
 
@@ -594,7 +659,13 @@ def main():
         v, nst, el = oracle_baseline(b, args.cpu_budget)
         cpu = {"value": v, "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"{nst} whole decode steps (append + attention over all {b.S} sequences) of the same "
-                         f"workload, single-threaded C fp64, {el:.1f} s"}
+                         f"workload, single-threaded C fp64, {el:.1f} s",
+               "cpu_model": cpu_model(), "affinity_cores": len(all_cores) if all_cores else None}
+        if all_cores and len(all_cores) > 1:
+            vp, nsp, elp, T = oracle_baseline_parallel(b, args.cpu_budget, all_cores)
+            cpu["all_cores"] = {"value": vp, "unit": "GB/s", "cores": T, "kind": "oracle",
+                                "sample": f"{nsp} whole decode steps, the attention's sequences over {T} threads "
+                                          f"(one per core; the append in place, on one), {elp:.1f} s"}
 
     traffic = None
     prof = os.path.join(ROOT, "profiles", "traffic.json")
