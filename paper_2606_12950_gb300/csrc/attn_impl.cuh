@@ -668,19 +668,25 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // waits for it at every exit (`chained`), so that a combine after it
     // sees every chained grid's records.  Data from earlier grids is then
     // read through L2 (ld_prior).  The first grid of a chain (chain 1)
-    // waits before it releases the next.
+    // waits before it releases the next.  With the lengths carried in the
+    // parameters (fused table sync) and no shared prefix, the first prologue
+    // below reads nothing that another grid writes and writes only shared
+    // memory, so a grid alone runs it before its wait, beside the grid
+    // before it (`early`).
+    const bool early = a.sync_table != nullptr && a.skip == nullptr && a.chain == 0;
     if (a.chain != 1) grid_launch_dependents();
-    if (a.chain != 2) grid_dependency_wait();
+    if (a.chain != 2 && !early) grid_dependency_wait();
     if (a.chain == 1) grid_launch_dependents();
     const bool chained = a.chain == 2;
-    if (a.sync_table) {
+    auto write_sync = [&]() {
         // fused table sync: the grids before have completed (the wait
-        // above), and no CTA of this grid reads what is written here
+        // before this), and no CTA of this grid reads what is written here
         const int stride = a.P * kThreads, i0 = (int)blockIdx.x * kThreads + tid;
         for (int i = i0; i < a.sync_nlens; i += stride) a.sync_lens[i] = a.sync_words[i];
         const int32_t *pw = a.sync_words + a.sync_nlens;
         for (int j = i0; j < a.sync_npatch; j += stride) a.sync_table[pw[2 * j]] = pw[2 * j + 1];
-    }
+    };
+    if (a.sync_table && !early) write_sync();
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {
@@ -695,17 +701,6 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             SK[s] = k;
             const int32_t ne = n - k;
             local += ((ne + kTile - 1) / kTile) * Hkv;
-            // the fused append needs the new token outside a shared prefix
-            if (ne == 0 && a.skip && a.k_new && n > 0 && (s % a.P) == (int)blockIdx.x)
-                report(a.err, KV_ERR_DEVICE_BOUNDS);
-            if (ne == 0 && (s % a.P) == (int)blockIdx.x) {
-                // an empty context has no softmax: its output is defined as
-                // zero; a sequence whose whole context is a shared prefix
-                // gets its output from the prefix records alone
-                if (n == 0)
-                    for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
-                for (int g = 0; g < Hkv; ++g) a.ws_run[(int64_t)s * Hkv + g] = make_int2(0, 0);
-            }
         }
         int32_t incl = local;
 #pragma unroll
@@ -726,6 +721,22 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             int32_t tot = 0;
             for (int w = 0; w < kWarps; ++w) tot += misc[w];
             T[S] = tot;
+        }
+        if (early) {
+            grid_dependency_wait();
+            write_sync();
+        }
+        for (int s = lo; s < hi; ++s) {  // sequences with no tile: writes after any wait
+            const int32_t n = NL[s] & 0x7fffffff, ne = n - SK[s];
+            if (ne != 0 || (s % a.P) != (int)blockIdx.x) continue;
+            // the fused append needs the new token outside a shared prefix
+            if (a.skip && a.k_new && n > 0) report(a.err, KV_ERR_DEVICE_BOUNDS);
+            // an empty context has no softmax: its output is defined as
+            // zero; a sequence whose whole context is a shared prefix gets
+            // its output from the prefix records alone
+            if (n == 0)
+                for (int i = 0; i < Hq * D; ++i) a.out[(int64_t)s * Hq * D + i] = 0;
+            for (int g = 0; g < Hkv; ++g) a.ws_run[(int64_t)s * Hkv + g] = make_int2(0, 0);
         }
         __syncthreads();
     }

@@ -66,7 +66,10 @@ int launch_chunk(kv_seqtab *t, int32_t *dev_table, int32_t *dev_lens, size_t li,
     return cudaLaunchKernelEx(&cfg, seqtab_sync_kernel<WORDS>, p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
+// parameter blocks of three sizes: a launch's cost grows with its parameter
+// bytes, so a sync takes the smallest block that holds it
 constexpr int kSmallWords = 256;
+constexpr int kMidWords = 1016;    // about 4 KB of parameters
 constexpr int kLargeWords = 4088;  // about 16 KB of parameters
 
 }  // namespace
@@ -97,6 +100,11 @@ extern "C" int kv_seqtab_sync(kv_seqtab *t, int32_t *dev_table, int32_t *dev_ctx
         if (want <= (size_t)kSmallWords) {
             const int nl = (int)(S - li), np = (int)(np_all - pi);
             rc = launch_chunk<kSmallWords>(t, dev_table, dev_ctx_lens, li, nl, pi, np, st);
+            li += (size_t)nl;
+            pi += (size_t)np;
+        } else if (want <= (size_t)kMidWords) {
+            const int nl = (int)(S - li), np = (int)(np_all - pi);
+            rc = launch_chunk<kMidWords>(t, dev_table, dev_ctx_lens, li, nl, pi, np, st);
             li += (size_t)nl;
             pi += (size_t)np;
         } else {
