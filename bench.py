@@ -224,6 +224,17 @@ def oracle_baseline_parallel(b, budget_s: float, cores):
 
 
 def cpu_model() -> str:
+    """The host CPU's model name (lscpu's, which names Arm cores too), else
+    /proc/cpuinfo's first model line, else the platform's."""
+    import subprocess
+
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
     try:
         with open("/proc/cpuinfo") as f:
             for line in f:
