@@ -320,7 +320,10 @@ int kv_seq_trim(kv_seqtab *t, int s);
  *                  left empty, length 0, and the admission is the caller's to
  *                  retry); the call itself still returns KV_OK
  * Every argument is checked before any slot changes: KV_ERR_INVALID_ARG and
- * nothing changed.  n = 0 is a no-op.
+ * nothing changed.  n = 0 is a no-op.  A failure of the pool itself while
+ * slots are replaced (a table naming blocks the pool does not hold live)
+ * returns that error at the slot where it occurred; the slots before it
+ * stay replaced.
  */
 int kv_seq_replace(kv_seqtab *t, int n, const int32_t *slots, const int64_t *reserve_tokens,
                    const int32_t *lens, int32_t *status);
