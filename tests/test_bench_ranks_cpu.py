@@ -73,3 +73,35 @@ def test_reference_arm_prints_on_rank0_only():
     line = json.loads(lines[0])
     assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_threaded_oracle_baseline_covers_every_sequence_once():
+    """The all-cores oracle timing computes the same attention as one
+    oracle call: the per-thread sequence subsets, merged, give the single
+    call's output exactly, and the timing helper runs on a small batch."""
+    sys.path.insert(0, ROOT)
+    import numpy as np
+
+    import bench
+    import oracle
+    from paper_2606_12950_gb300 import workloads as W
+
+    b = W.make_batch(31, [5, 40, 17, 1, 64, 33, 9], Hq=4, Hkv=2, d=16, bs=4, extra_blocks=8)
+    full = oracle.paged_attention(b.pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q, b.table,
+                                  b.ctx_lens, b.scale)
+    T = 3
+    order = np.argsort(-b.ctx_lens.astype(np.int64), kind="stable")
+    merged = np.full_like(full, np.nan)
+    for i in range(T):
+        ids = order[i::T].astype(np.int32)
+        part = oracle.paged_attention(b.pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q, b.table,
+                                      b.ctx_lens, b.scale, seq_ids=ids)
+        assert np.isnan(part[np.setdiff1d(np.arange(b.S), ids)]).all()
+        merged[ids] = part[ids]
+    assert np.array_equal(merged, full)
+    b.meta["seed"] = 31
+    cores = set(sorted(os.sched_getaffinity(0))[:2])
+    before = os.sched_getaffinity(0)
+    gbs, steps, el, threads = bench.oracle_baseline_parallel(b, 0.0, cores)
+    assert steps == 1 and gbs > 0 and threads == len(cores)
+    assert os.sched_getaffinity(0) == before  # the caller's affinity is restored
