@@ -37,7 +37,8 @@
 // a chain (beside the shared-prefix kernel, or the later batches of several
 // co-located ones) it starts without waiting, reads what earlier grids wrote
 // through L2 only, and waits at its end (AttnArgs::chain).  The step's
-// table sync may ride in its parameters (AttnArgs::sync_words).
+// table sync may ride in its parameters (AttnArgs::sync_words); a grid
+// alone then computes its work split from those lengths before its wait.
 //
 // Two compute variants share this skeleton:
 //   FmaCompute : CUDA-core FFMA2 dot products and weighted sums.
