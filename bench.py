@@ -146,50 +146,70 @@ def aggregate_ranks(dist, device, ms: float, e2e_ms: float, units: dict) -> tupl
     return tl[0], tl[1], dict(zip(keys, ul))
 
 
-def oracle_baseline(b, budget_s: float):
+def oracle_lap_steps(b) -> int:
+    """How many consecutive decode steps the batch's fixed table holds from
+    its step-0 lengths: step i appends at position ctx_lens + i - 1, which
+    must fall inside the blocks the table row lists.  At least 1."""
+    cap = (b.table >= 0).sum(axis=1).astype(np.int64) * b.bs
+    return max(1, int((cap - b.ctx_lens.astype(np.int64)).min()) + 1)
+
+
+def _step_bytes(b, lens) -> int:
+    kv = int(lens.astype(np.int64).sum()) * 2 * b.Hkv * b.d * 2
+    return kv + 2 * b.S * b.Hq * b.d * 2 + 2 * b.S * b.Hkv * b.d * 2
+
+
+def oracle_baseline(b, budget_s: float, max_steps: int = 1000):
     """Time the fp64 C oracle (single thread) on whole decode steps of the
     same workload (append + attention over every sequence) until budget_s
-    elapses; return (GB/s of algorithmic bytes, steps, seconds)."""
+    elapses or max_steps steps are done; return (GB/s of algorithmic bytes,
+    steps, seconds).  The steps run in laps of at most oracle_lap_steps(b):
+    each lap starts again from the step-0 pool and lengths (untimed), so an
+    append never leaves the table's reserved blocks however fast the host
+    is, and the lengths follow the same schedule as the GPU arm's steps."""
     import oracle
 
     oracle.build()
-    pool = b.pool
-    lens = b.ctx_lens.copy()
-    t0 = time.perf_counter()
+    lap = oracle_lap_steps(b)
+    el = 0.0
     done_bytes = 0
     steps = 0
     while True:
-        q, kn, vn = W_step_rows(b, steps)
-        pool = oracle.append(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens)
-        oracle.paged_attention(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, q, b.table, lens, b.scale)
-        kv = int(lens.astype(np.int64).sum()) * 2 * b.Hkv * b.d * 2
-        done_bytes += kv + 2 * b.S * b.Hq * b.d * 2 + 2 * b.S * b.Hkv * b.d * 2
-        steps += 1
-        lens = lens + 1
-        el = time.perf_counter() - t0
-        if el >= budget_s or steps >= 1000:
-            return done_bytes / el / 1e9, steps, el
+        pool = b.pool
+        lens = b.ctx_lens.copy()
+        for i in range(lap):
+            t0 = time.perf_counter()
+            q, kn, vn = W_step_rows(b, i)
+            pool = oracle.append(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens)
+            oracle.paged_attention(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, q, b.table, lens, b.scale)
+            el += time.perf_counter() - t0
+            done_bytes += _step_bytes(b, lens)
+            steps += 1
+            lens = lens + 1
+            if el >= budget_s or steps >= max_steps:
+                return done_bytes / el / 1e9, steps, el
 
 
-def oracle_baseline_parallel(b, budget_s: float, cores):
+def oracle_baseline_parallel(b, budget_s: float, cores, max_steps: int = 1000):
     """The same whole decode steps as oracle_baseline, with each step's
     attention spread over one thread per core: thread i computes the
     sequences at ranks i, i + T, ... of a longest-first order (the oracle's
     own seq_ids subset; ctypes releases the interpreter lock during the C
     call, so the threads run at once).  The append writes the pool in place
     (the oracle's inplace option) instead of into a fresh copy of it; the
-    oracle's arithmetic is unchanged.  Returns (GB/s, steps, seconds,
-    threads)."""
+    oracle's arithmetic is unchanged.  Laps as in oracle_baseline: between
+    laps the pool is copied back from the step-0 pool outside the timed
+    steps.  Returns (GB/s, steps, seconds, threads)."""
     from concurrent.futures import ThreadPoolExecutor
 
     import oracle
 
     oracle.build()
     T = max(1, len(cores))
+    lap = oracle_lap_steps(b)
     order = np.argsort(-b.ctx_lens.astype(np.int64), kind="stable")
     subsets = [order[i::T].astype(np.int32) for i in range(T)]
     pool = np.array(b.pool, dtype=np.uint16, copy=True)  # appended in place below
-    lens = b.ctx_lens.copy()
     try:
         before = os.sched_getaffinity(0)
         os.sched_setaffinity(0, cores)  # threads created below inherit every core
@@ -197,22 +217,30 @@ def oracle_baseline_parallel(b, budget_s: float, cores):
         before = None
     try:
         with ThreadPoolExecutor(T) as ex:
-            t0 = time.perf_counter()
+            el = 0.0
             done_bytes = 0
             steps = 0
-            while True:
-                q, kn, vn = W_step_rows(b, steps)
-                oracle.append(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens, inplace=True)
-                outs = list(ex.map(lambda ids: oracle.paged_attention(pool, b.n_pages, b.page_elems, b.bs, b.Hkv,
-                                                                      b.d, q, b.table, lens, b.scale, seq_ids=ids),
-                                   subsets))
-                kv = int(lens.astype(np.int64).sum()) * 2 * b.Hkv * b.d * 2
-                done_bytes += kv + 2 * b.S * b.Hq * b.d * 2 + 2 * b.S * b.Hkv * b.d * 2
-                steps += 1
-                lens = lens + 1
-                el = time.perf_counter() - t0
-                if el >= budget_s or steps >= 1000:
-                    break
+            finished = False
+            while not finished:
+                if steps:
+                    np.copyto(pool, b.pool)  # back to the step-0 pool (untimed)
+                lens = b.ctx_lens.copy()
+                for i in range(lap):
+                    t0 = time.perf_counter()
+                    q, kn, vn = W_step_rows(b, i)
+                    oracle.append(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, kn, vn, b.table, lens,
+                                  inplace=True)
+                    outs = list(ex.map(lambda ids: oracle.paged_attention(pool, b.n_pages, b.page_elems, b.bs,
+                                                                          b.Hkv, b.d, q, b.table, lens, b.scale,
+                                                                          seq_ids=ids),
+                                       subsets))
+                    el += time.perf_counter() - t0
+                    done_bytes += _step_bytes(b, lens)
+                    steps += 1
+                    lens = lens + 1
+                    if el >= budget_s or steps >= max_steps:
+                        finished = True
+                        break
     finally:
         if before is not None:
             os.sched_setaffinity(0, before)

@@ -8,6 +8,7 @@ import socket
 import subprocess
 import sys
 
+import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")
@@ -105,3 +106,41 @@ def test_threaded_oracle_baseline_covers_every_sequence_once():
     gbs, steps, el, threads = bench.oracle_baseline_parallel(b, 0.0, cores)
     assert steps == 1 and gbs > 0 and threads == len(cores)
     assert os.sched_getaffinity(0) == before  # the caller's affinity is restored
+
+
+def test_oracle_baselines_run_past_the_table_headroom():
+    """Both oracle timings run more steps than the batch's table holds: the
+    steps go in laps from the step-0 state, so no append leaves the
+    reserved blocks (the fixed table holds 3 more appends here), and every
+    lap's lengths are the step-0 lengths plus the lap's step index."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2606_12950_gb300 import workloads as W
+
+    pre = [5, 40, 17, 1, 64, 33, 9]
+    b = W.make_batch(37, pre, Hq=4, Hkv=2, d=16, bs=4, extra_blocks=8,
+                     table_tokens=[p + 3 for p in pre])
+    b.meta["seed"] = 37
+    lap = bench.oracle_lap_steps(b)
+    cap = (b.table >= 0).sum(axis=1) * b.bs
+    assert lap == int((cap - b.ctx_lens).min()) + 1 and 1 <= lap <= 4
+    gbs, steps, el = bench.oracle_baseline(b, 1e9, max_steps=5 * lap + 2)
+    assert steps == 5 * lap + 2 and gbs > 0
+    cores = set(sorted(os.sched_getaffinity(0))[:2])
+    gbs, steps, el, threads = bench.oracle_baseline_parallel(b, 1e9, cores, max_steps=5 * lap + 2)
+    assert steps == 5 * lap + 2 and gbs > 0 and threads == len(cores)
+
+
+def test_oracle_baseline_on_the_benchmark_batch_at_the_driver_step_counts():
+    """The benchmark's own batch at 20 steps + 5 warm-up: the oracle's
+    laps fit its table however many steps the time budget allows."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2606_12950_gb300 import workloads as W
+
+    b = W.config2_llama8b(steps=max(100, 2 * (5 + 20) + 8), fill_pool=False)
+    lap = bench.oracle_lap_steps(b)
+    cap = (b.table >= 0).sum(axis=1) * b.bs
+    for i in range(lap):  # every appended position of a lap is inside its row's blocks
+        assert np.all(b.ctx_lens + i - 1 < cap)
+    assert np.any(b.ctx_lens + lap - 1 >= cap)
