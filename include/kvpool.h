@@ -632,11 +632,17 @@ int paged_decode_attn_cascade(kv_pool *pool, int layout, const uint16_t *q, cons
  * device) is not acceptable.
  * Arguments and results are those of paged_decode_attn without the
  * workspace.  The split-K scratch is instead a fixed 32 MiB device array
- * inside the library, which every GPU that loads the library holds until
- * the process exits.  The call allocates nothing.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call
+ * inside the library, held on a device until the process exits once it has
+ * been taken there.  The call allocates nothing.
+ *   - Creating a pool (kv_pool_create, kv_pool_create_vmm) looks up the
+ *     array's device address (cudaGetSymbolAddress) with the pool's device
+ *     current.  CUDA loads modules lazily by default, so that lookup is when
+ *     the 32 MiB are taken from the device: before the caller fills the
+ *     device with KV blocks.  If it failed there, the first call on the
+ *     device repeats it, and then needs the 32 MiB free.  Create the pool
  *     before any stream capture.
+ *   - The pool's device must be the current device (else
+ *     KV_ERR_INVALID_ARG, nothing launched): each device has its own array.
  *   - If kv_workspace_bytes for the same arguments exceeds 32 MiB the call
  *     returns KV_ERR_WORKSPACE and launches nothing; use paged_decode_attn
  *     with a workspace for such batches.

@@ -11,7 +11,7 @@
 
 #include <cuda_runtime.h>
 
-#include "kvpool.h"
+#include "pool_internal.h"
 
 namespace {
 
@@ -20,7 +20,8 @@ namespace {
 // process exits.
 constexpr size_t kScratchBytes = 32u << 20;  // 32 MiB
 
-// Per-device address of the scratch array, resolved on first use.
+// Per-device address of the scratch array, resolved when a pool is created
+// on the device (kvp_noalloc_prepare) or else on the first call.
 constexpr int kMaxDevices = 64;
 void *g_scratch_addr[kMaxDevices] = {};
 std::mutex g_scratch_mu;
@@ -33,16 +34,22 @@ static __device__ __align__(256) unsigned char g_attn_scratch[kScratchBytes];
 
 namespace {
 
-// Resolve the scratch address for the current device (once per device).
-int scratch_for_current_device(void **out)
+// Resolve the scratch address of device `dev`, which must be the current
+// device (once per device).  The lookup loads the module that holds the
+// array if it is not loaded yet (CUDA loads modules lazily by default), and
+// that is when the array's 32 MiB are taken from the device.  On failure
+// the runtime's last-error slot is cleared, so that the failure is not
+// reported again by an unrelated later call on this thread.
+int scratch_for_device(int dev, void **out)
 {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return KV_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return KV_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> g(g_scratch_mu);
     if (!g_scratch_addr[dev]) {
         void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_attn_scratch) != cudaSuccess || !p) return KV_ERR_CUDA;
+        if (cudaGetSymbolAddress(&p, g_attn_scratch) != cudaSuccess || !p) {
+            cudaGetLastError();
+            return KV_ERR_CUDA;
+        }
         g_scratch_addr[dev] = p;
     }
     *out = g_scratch_addr[dev];
@@ -50,6 +57,16 @@ int scratch_for_current_device(void **out)
 }
 
 }  // namespace
+
+// Called by kv_pool_create with the pool's device current: takes the
+// scratch array's memory on that device before the caller fills the device
+// with KV blocks, so a later first noalloc call needs no device memory.  A
+// failure here is not an error of the pool; the first call retries.
+void kvp_noalloc_prepare(int device)
+{
+    void *p = nullptr;
+    (void)scratch_for_device(device, &p);
+}
 
 extern "C" {
 
@@ -61,8 +78,16 @@ int paged_decode_attn_noalloc(kv_pool *pool, int layout, const uint16_t *q, uint
     int rc = kv_workspace_bytes(pool, layout, S, Hq, max_blocks, num_splits, &need);
     if (rc) return rc;
     if (need > kScratchBytes) return KV_ERR_WORKSPACE;  // batch too large for the fixed scratch
+    // the scratch used must be the one on the pool's device, which is where
+    // the kernels launch: the pool's device has to be the current one
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return KV_ERR_CUDA;
+    }
+    if (dev != pool->device) return KV_ERR_INVALID_ARG;
     void *scratch = nullptr;
-    rc = scratch_for_current_device(&scratch);
+    rc = scratch_for_device(dev, &scratch);
     if (rc) return rc;
     return paged_decode_attn(pool, layout, q, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale, num_splits,
                              scratch, kScratchBytes, stream);

@@ -112,6 +112,10 @@ int kv_pool_create(const kv_pool_desc *desc, kv_pool **out_pool)
         // host-only use (no GPU visible): allocation still works; launches will fail
         cudaGetLastError();
         p->sm_count = 0;
+    } else {
+        // the allocation-free attention's fixed scratch is taken on this
+        // device now, before the caller fills it with KV blocks
+        kvp_noalloc_prepare(p->device);
     }
     *out_pool = p;
     return KV_OK;

@@ -66,6 +66,10 @@ void kvp_vmm_release_all(kv_pool *p);                // on destroy
 // table still open over the pool (seqtab.cpp).
 void kvp_seqtab_detach(kv_seqtab *t);
 
+// Resolve the allocation-free attention's scratch on `device`, the current
+// device (noalloc.cu); called when a pool is created on a visible GPU.
+void kvp_noalloc_prepare(int device);
+
 // Validate that a block id is a whole block of layout L inside the pool.
 // In a VMM pool the block must also lie in a mapped chunk.
 inline bool kvp_block_in_pool(const kv_pool *p, int layout, int64_t id)
