@@ -422,6 +422,12 @@ class Coloc:
                               b.v_new, args.num_splits)
             K.kv_block_table_upload(self.pool.handle, li, b.table, b.ctx_lens, buf.table, buf.lens)
             self.bufs.append(buf)
+        only = getattr(args, "layout", None)
+        if only is not None:
+            # one co-located layout's batch alone, in the same 90%-full pool
+            # (its per-layout figures; the step is then that batch's call)
+            batches, self.bufs = [batches[only]], [self.bufs[only]]
+            self.name += f"; layout {only} alone"
         self.batches = batches
         self.S = sum(b.S for b in batches)
         self.config = {"S": self.S, "layouts": [[b.Hq, b.Hkv, b.d] for b in batches], "bs": 16,
@@ -493,6 +499,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
+    ap.add_argument("--layout", type=int, default=None, choices=[0, 1, 2],
+                    help="coloc: time one co-located layout's batch alone (0 MHA 32/32, 1 GQA 32/8, 2 GQA 40/8)")
     ap.add_argument("--separate-batches", action="store_true",
                     help="one call per co-located batch instead of one paged_decode_attn_multi call")
     ap.add_argument("--separate-sync", action="store_true",
