@@ -59,8 +59,14 @@
 
 namespace kvp {
 
-constexpr int kWarps = 8;  // each warp streams and computes its own units
+// Warps per CTA, each streaming and computing its own units: up to kWarps
+// (AttnArgs::nwarps).  Two CTAs of six warps on an SM keep 12 units in
+// flight there, which config 2 (64 sequences on all 152 SMs) streams
+// fastest; beside the shared-prefix kernel, on fewer SMs, eight do.
+constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
+constexpr int kPlainWarps = 6;
+constexpr int kStages = 1;  // units in flight per warp (each a K and a V tile)
 constexpr int kTile = 16;                         // tokens per unit
 constexpr int kMinUnitsPerPart = 4;
 constexpr uint32_t kHalfBytes = kTile * 128;      // one 64-column box: 16 rows x 128 B
@@ -101,7 +107,8 @@ struct AttnArgs {
     int32_t Hkv;
     int32_t bs;
     int32_t rows_cap;        // units whose pool rows are resolved up front
-    int32_t P;               // CTAs (work partitions)
+    int32_t P;               // CTAs
+    int32_t nwarps;          // warps per CTA (<= kWarps), one part each
     float qk_scale;          // scale * log2(e)
     // shared-prefix (cascade) mode: tokens of each sequence's prefix handled
     // by the prefix kernel ([S], multiples of 16; null = none), its records
@@ -640,11 +647,12 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // stages need 1024-byte alignment for the 128-byte swizzle pattern
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     constexpr uint32_t QB = G * D * 2, AB = 2 * D * 2;  // q rows of a run; its new K and V rows
-    uint8_t *stages = smem;                                                              // [kWarps][STAGE]
-    uint8_t *qbufs = stages + (size_t)kWarps * STAGE_BYTES;                              // [kWarps][QB]
-    uint8_t *abufs = qbufs + (size_t)kWarps * QB;                                        // [kWarps][AB]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(abufs + (size_t)kWarps * AB);          // K[w], V[w]
-    int32_t *misc = reinterpret_cast<int32_t *>(bars + 2 * kWarps);                     // [16] scratch
+    const int NW = a.nwarps, NT = NW * 32;  // warps (parts) of this CTA
+    uint8_t *stages = smem;                                                              // [NW][kStages][STAGE]
+    uint8_t *qbufs = stages + (size_t)NW * kStages * STAGE_BYTES;                        // [NW][QB]
+    uint8_t *abufs = qbufs + (size_t)NW * QB;                                            // [NW][AB]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(abufs + (size_t)NW * AB);              // K[w][st], V[w][st]
+    int32_t *misc = reinterpret_cast<int32_t *>(bars + 2 * NW * kStages);               // [16] scratch
     int32_t *T = misc + 16;                                                              // [S + 1]
     int32_t *NL = T + a.S + 1;                                                           // [S]
     int32_t *SK = NL + a.S;                                                              // [S]
@@ -654,7 +662,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     const int S = a.S, Hkv = a.Hkv, Hq = a.Hkv * G;
 
     if (tid == 0) {
-        for (int i = 0; i < 2 * kWarps; ++i) mbar_init(smem_u32(&bars[i]), 1);
+        for (int i = 0; i < 2 * NW * kStages; ++i) mbar_init(smem_u32(&bars[i]), 1);
         fence_mbar_init();
     }
     if (tid == 32) prefetch_tensormap(&tmap);
@@ -682,7 +690,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     auto write_sync = [&]() {
         // fused table sync: the grids before have completed (the wait
         // before this), and no CTA of this grid reads what is written here
-        const int stride = a.P * kThreads, i0 = (int)blockIdx.x * kThreads + tid;
+        const int stride = a.P * NT, i0 = (int)blockIdx.x * NT + tid;
         for (int i = i0; i < a.sync_nlens; i += stride) a.sync_lens[i] = a.sync_words[i];
         const int32_t *pw = a.sync_words + a.sync_nlens;
         for (int j = i0; j < a.sync_npatch; j += stride) a.sync_table[pw[2 * j]] = pw[2 * j + 1];
@@ -691,7 +699,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
 
     // ---- prologue 1: T[s] = first unit of sequence s ----
     {
-        const int per = (S + kThreads - 1) / kThreads;
+        const int per = (S + NT - 1) / NT;
         const int lo = min(S, tid * per), hi = min(S, lo + per);
         int32_t local = 0;
         for (int s = lo; s < hi; ++s) {
@@ -720,7 +728,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         }
         if (tid == 0) {
             int32_t tot = 0;
-            for (int w = 0; w < kWarps; ++w) tot += misc[w];
+            for (int w = 0; w < NW; ++w) tot += misc[w];
             T[S] = tot;
         }
         if (early) {
@@ -742,21 +750,21 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         __syncthreads();
     }
 
-    // The W units are cut into NP = min(P * kWarps, W) equal parts; part i is
-    // [i*W/NP, (i+1)*W/NP) and belongs to warp i % kWarps of CTA i / kWarps.
+    // The W units are cut into NP = min(P * NW, W) equal parts; part i is
+    // [i*W/NP, (i+1)*W/NP) and belongs to warp i % NW of CTA i / NW.
     // With NP <= W every part is non-empty, so a run's contributors are
     // exactly the parts part_of(first unit) .. part_of(last unit).  A part
     // gets at least kMinUnitsPerPart units when the batch is small (fewer
     // partials to write and merge; enough warps still stream to fill HBM).
     const int64_t W = T[S];
     const int64_t np_min = W > 0 ? (W / kMinUnitsPerPart > 0 ? W / kMinUnitsPerPart : 1) : 0;
-    const int64_t NP = np_min < (int64_t)a.P * kWarps ? np_min : (int64_t)a.P * kWarps;
-    const int64_t first_part = (int64_t)blockIdx.x * kWarps;
+    const int64_t NP = np_min < (int64_t)a.P * NW ? np_min : (int64_t)a.P * NW;
+    const int64_t first_part = (int64_t)blockIdx.x * NW;
     if (first_part >= NP) {
         if (chained) grid_dependency_wait();
         return;
     }
-    const int64_t last_part = first_part + kWarps < NP ? first_part + kWarps : NP;  // exclusive
+    const int64_t last_part = first_part + NW < NP ? first_part + NW : NP;  // exclusive
     const int32_t cu0 = (int32_t)(first_part * W / NP);                             // this CTA's units
     const int32_t cu1 = (int32_t)(last_part * W / NP);
 
@@ -764,7 +772,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // memory system is idle (later lookups would queue behind the TMA stream)
     {
         const int32_t nr = min(cu1 - cu0, a.rows_cap);
-        for (int32_t k = tid; k < nr; k += kThreads) rows[k] = unit_row(a, T, cu0 + k);
+        for (int32_t k = tid; k < nr; k += NT) rows[k] = unit_row(a, T, cu0 + k);
         __syncthreads();
     }
 
@@ -777,14 +785,17 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     const int32_t u1 = (int32_t)((part + 1) * W / NP);
 
     const uint64_t policy = l2_policy_evict_first();
-    uint8_t *Ks = stages + (size_t)warp * STAGE_BYTES;
-    uint8_t *Vs = Ks + TILE_BYTES;
-    const uint32_t k_addr = smem_u32(Ks), v_addr = smem_u32(Vs);
-    const uint32_t bk = smem_u32(&bars[warp]), bv = smem_u32(&bars[kWarps + warp]);
+    // stage st of this warp: its K and V tiles and their barriers
+    uint8_t *wstage = stages + (size_t)warp * kStages * STAGE_BYTES;
+    auto k_of = [&](int st) { return wstage + (size_t)st * STAGE_BYTES; };
+    auto bk_of = [&](int st) { return smem_u32(&bars[warp * kStages + st]); };
+    auto bv_of = [&](int st) { return smem_u32(&bars[(NW + warp) * kStages + st]); };
 
     if (lane == 0) {
-        issue_half<D>(&tmap, a, T, rows, cu0, u0, 0, k_addr, bk, policy);
-        issue_half<D>(&tmap, a, T, rows, cu0, u0, 1, v_addr, bv, policy);
+        for (int st = 0; st < kStages && u0 + st < u1; ++st) {
+            issue_half<D>(&tmap, a, T, rows, cu0, u0 + st, 0, smem_u32(k_of(st)), bk_of(st), policy);
+            issue_half<D>(&tmap, a, T, rows, cu0, u0 + st, 1, smem_u32(k_of(st) + TILE_BYTES), bv_of(st), policy);
+        }
     }
     // A run's q rows and, for the run's last tile, its new K/V rows are staged
     // in this warp's shared buffers by cp.async one piece ahead, so that no
@@ -826,9 +837,13 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         }
         cp_async_commit();
         for (int32_t uu = pc.pb; uu < pc.pe; ++uu) {
-            const uint32_t par = consumed & 1u;
+            const int st = (int)(consumed % kStages);
+            const uint32_t par = (consumed / kStages) & 1u;
+            uint8_t *Ks = k_of(st);
+            uint8_t *Vs = Ks + TILE_BYTES;
+            const uint32_t bk = bk_of(st), bv = bv_of(st);
             const int nvalid = min(kTile, pc.n - pc.skip - (uu - pc.run_begin) * kTile);
-            const bool more = uu + 1 < u1;
+            const bool more = uu + kStages < u1;  // the unit this stage takes next
             const bool app = app_run && uu == pc.run_end - 1;
             const int arow = (pc.n - 1) % kTile;
             wait_phase(bk, par, a.err, dead);
@@ -844,7 +859,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             // shared-memory reads before the async-proxy write
             fence_proxy_async_smem();
             __syncwarp();
-            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 0, k_addr, bk, policy);
+            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + kStages, 0, smem_u32(Ks), bk, policy);
             wait_phase(bv, par, a.err, dead);
             if (app) {
                 if (lane < D / 8)
@@ -867,7 +882,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + 1, 1, v_addr, bv, policy);
+            if (more && lane == 0) issue_half<D>(&tmap, a, T, rows, cu0, uu + kStages, 1, smem_u32(Vs), bv, policy);
             ++consumed;
         }
 
@@ -1022,15 +1037,16 @@ __global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __gri
 constexpr int kRowsCap = 2048;
 
 template <int D, int G>
-inline size_t attn_smem_bytes(int S, int rows_cap)
+inline size_t attn_smem_bytes(int S, int rows_cap, int nwarps)
 {
     const size_t stage = 2ull * (D / 64) * kHalfBytes;
     const size_t bufs = (size_t)G * D * 2 + 2 * D * 2;  // per warp: q rows, new K/V rows
-    return 1024 + (size_t)kWarps * (stage + bufs) + (2 * kWarps) * 8 + 64 + (size_t)(3 * S + 1) * 4 +
+    return 1024 + (size_t)nwarps * (kStages * stage + bufs) + (2 * nwarps * kStages) * 8 + 64 + (size_t)(3 * S + 1) * 4 +
            (size_t)rows_cap * 4;
 }
 
-// partial records: one per (run, part) pair that a run can touch
+// partial records: one per (run, part) pair that a run can touch (parts:
+// at most kWarps per CTA)
 inline size_t attn_partial_slots(int S, int Hkv, int P) { return (size_t)S * Hkv + (size_t)P * kWarps; }
 
 }  // namespace kvp

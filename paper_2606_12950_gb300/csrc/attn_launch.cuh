@@ -15,21 +15,32 @@ namespace kvp {
 constexpr size_t kSmemMax = 227 * 1024;
 
 // Resident CTAs per SM of kernel fn at this block size and dynamic shared
-// memory, queried once per (instantiation, shared-memory size) and cached:
-// the runtime query costs microseconds of host time on every launch.
+// memory, queried once per (block size, shared-memory size) and cached in
+// the caller's slot, one slot per kernel instantiation: the runtime query
+// costs microseconds of host time on every launch.
+struct OccCache {
+    static constexpr int kSlots = 4;  // a call may query two shapes (its workspace's, its launch's)
+    // (smem * 2048 + threads) << 8 | CTAs per SM, one word so that a reader
+    // sees a key only with its own value
+    std::atomic<long long> slot[kSlots] = {{-1}, {-1}, {-1}, {-1}};
+    std::atomic<unsigned> next{0};
+};
+
 template <class Fn>
-int cached_occupancy(Fn fn, int threads, size_t smem, int *occ)
+int cached_occupancy(Fn fn, int threads, size_t smem, int *occ, OccCache &c)
 {
-    static std::atomic<long long> key{-1};
-    static std::atomic<int> val{0};
-    if (key.load(std::memory_order_acquire) == (long long)smem) {
-        *occ = val.load(std::memory_order_relaxed);
-        return KV_OK;
+    const long long key = (long long)smem * 2048 + threads;
+    for (int i = 0; i < OccCache::kSlots; ++i) {
+        const long long w = c.slot[i].load(std::memory_order_relaxed);
+        if (w >= 0 && (w >> 8) == key) {
+            *occ = (int)(w & 255);
+            return KV_OK;
+        }
     }
     int o = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, threads, smem) != cudaSuccess) return KV_ERR_CUDA;
-    val.store(o, std::memory_order_relaxed);
-    key.store((long long)smem, std::memory_order_release);
+    const unsigned i = c.next.fetch_add(1, std::memory_order_relaxed) % OccCache::kSlots;
+    c.slot[i].store(key << 8 | (long long)(o & 255), std::memory_order_relaxed);
     *occ = o;
     return KV_OK;
 }
@@ -48,10 +59,13 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
             return KV_ERR_CUDA;
         attr_set.store(true);
     }
-    const size_t smem = attn_smem_bytes<D, G>(a.S, kRowsCap);
+    // six warps a CTA, eight beside the shared-prefix kernel (kPlainWarps)
+    a.nwarps = a.skip != nullptr ? kWarps : kPlainWarps;
+    const size_t smem = attn_smem_bytes<D, G>(a.S, kRowsCap, a.nwarps);
     if (smem > kSmemMax) return KV_ERR_INVALID_ARG;  // S too large for the per-CTA sequence index
     int occ = 0;
-    if (cached_occupancy(fn, kThreads, smem, &occ) != KV_OK) return KV_ERR_CUDA;
+    static OccCache occ_cache;
+    if (cached_occupancy(fn, a.nwarps * 32, smem, &occ, occ_cache) != KV_OK) return KV_ERR_CUDA;
     const int P = P_req > 0 ? P_req : std::max(1, occ) * std::max(1, sm_count);
     *P_out = P;
     if (what == kLaunchQuery) return KV_OK;
@@ -65,7 +79,7 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)P);
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3((unsigned)(a.nwarps * 32));
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cfg.attrs = attr;
@@ -74,9 +88,9 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     if (what == kLaunchAttention) return KV_OK;
     CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv, a.skip, a.ws_pre, a.KS};
     cudaLaunchConfig_t ccfg = cfg;
-    // records per run: at most P * kWarps parts spread over the runs, plus
+    // records per run: at most P * nwarps parts spread over the runs, plus
     // the prefix records in shared-prefix mode
-    const double per_run = (double)P * kWarps / std::max(1, a.S * a.Hkv) + 1.0 + (a.skip ? a.KS : 0);
+    const double per_run = (double)P * a.nwarps / std::max(1, a.S * a.Hkv) + 1.0 + (a.skip ? a.KS : 0);
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv));
     ccfg.blockDim = dim3((unsigned)(combine_groups<D, G>(per_run, a.skip != nullptr) * (G * D / 4)));
     ccfg.dynamicSmemBytes = 0;
@@ -100,7 +114,8 @@ int cascade_run(const CUtensorMap *tmap, const CascadeArgs *c, int grid, int sm_
     }
     if (!launch) {
         int occ = 0;
-        if (cached_occupancy(fn, kPreThreads, smem, &occ) != KV_OK) return KV_ERR_CUDA;
+        static OccCache occ_cache;
+        if (cached_occupancy(fn, kPreThreads, smem, &occ, occ_cache) != KV_OK) return KV_ERR_CUDA;
         *P_out = std::max(1, occ) * std::max(1, sm_count);
         return KV_OK;
     }
