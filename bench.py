@@ -487,6 +487,108 @@ W_PREFIX = 2048
 WORKLOADS = {"llama8b": Llama8B, "chains": Chains, "coloc": Coloc, "longctx": LongCtx}
 
 
+class StepRunner:
+    """One decode step of a workload through the library's calls: the host
+    bookkeeping, the table sync (carried by the decode launch when it fits),
+    then append + attention per batch, by the call the options select."""
+
+    def __init__(self, wl, args, K, stream):
+        self.wl, self.args, self.K, self.stream = wl, args, K, stream
+        self.launches_per_step = 0
+        self.cascade = None
+        if hasattr(wl, "prefix_plan") and not args.no_cascade and not args.separate_append:
+            self.cascade = wl.prefix_plan()
+            for _, buf in wl.tables():
+                buf.use_cascade()
+        self.fuse_sync = self.cascade is None and not args.separate_append and not args.separate_sync
+        # co-located batches without host tables (the same step repeated): one call
+        self.multi = (self.cascade is None and not args.separate_append and not args.separate_batches
+                      and len(wl.tables()) > 1 and all(tab is None for tab, _ in wl.tables()))
+
+    def sync_kernels(self):
+        return sum(tab.counters()["sync_launches"] for tab, _ in self.wl.tables() if tab is not None)
+
+    def step(self, ev_pair=None):
+        """host bookkeeping, table sync, then append + attention per batch;
+        returns the step's (DRAM-algorithmic, logical) bytes"""
+        wl, args, K, stream = self.wl, self.args, self.K, self.stream
+        nbytes = wl.host_step()
+        n = 0
+        if not self.fuse_sync:
+            for tab, buf in wl.tables():
+                if tab is not None:
+                    tab.sync(buf.table, buf.lens, stream)
+                    n += 1
+        if ev_pair is not None:
+            ev_pair[0].record(stream)
+        if self.multi:
+            # every batch's decode kernel as one chain, then the combines
+            K.paged_decode_attn_multi(wl.pool.handle, [buf.batch() for _, buf in wl.tables()], stream)
+            n += 2 * len(wl.tables())
+        for tab, buf in (() if self.multi else wl.tables()):
+            if self.fuse_sync and tab is not None:
+                # table sync, append and attention: the decode launch carries
+                # the sync when it fits (else a sync kernel runs first; those
+                # launches are counted from the tables' counters)
+                buf.sync_append_attend(tab, stream)
+                n += 2
+            elif self.cascade is not None:
+                buf.cascade(self.cascade, stream=stream)  # plan, attention (fused append), prefix kernel, combine
+                n += 4
+            elif args.separate_append:
+                buf.append(stream)
+                buf.attend(stream)
+                n += 3
+            else:
+                buf.append_attend(stream)  # the append fused into the attention pass
+                n += 2
+        if ev_pair is not None:
+            ev_pair[1].record(stream)
+        self.launches_per_step = n
+        return nbytes
+
+
+def measure_secondary(name, args, K, W, DevicePool, DeviceSteps, stream, peak):
+    """The step of another workload (agent chains, co-location, long
+    context), timed like the main one over min(steps, 30) steps after a
+    short warm-up (device-resident inputs, CUDA events around the region);
+    its buffers are freed afterwards."""
+    import torch
+
+    sargs = argparse.Namespace(**vars(args))
+    sargs.workload = name
+    wl = WORKLOADS[name](sargs, K, W, DevicePool, DeviceSteps)
+    run = StepRunner(wl, sargs, K, stream)
+    steps = max(1, min(args.steps, 30))
+    gc.collect()
+    gc.freeze()
+    gc.disable()
+    for _ in range(max(3, min(args.warmup, 5))):
+        run.step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    nb = [run.step() for _ in range(steps)]
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    dram = sum(x[0] for x in nb) / steps
+    logical = sum(x[1] for x in nb) / steps
+    res = {"workload": wl.name, "steps": steps, "ms_per_step": ms, "gbs": dram / (ms * 1e-3) / 1e9,
+           "frac_of_peak": dram / (ms * 1e-3) / 1e9 / peak, "decode_tokens_per_s": wl.S / (ms * 1e-3),
+           "device_error": wl.pool.error(stream)}
+    if logical != dram:
+        res["logical_gbs"] = logical / (ms * 1e-3) / 1e9
+    del run
+    wl.pool.close()
+    del wl
+    gc.enable()
+    gc.collect()
+    torch.cuda.empty_cache()
+    return res
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -498,6 +600,8 @@ def main():
     ap.add_argument("--variant", type=int, default=0, help="0 auto, 1 CUDA cores, 2 tensor-core MMA")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle time for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="llama8b: skip timing the agent-chains, co-location and long-context steps too")
     ap.add_argument("--separate-append", action="store_true", help="append with its own kernel (unfused)")
     ap.add_argument("--layout", type=int, default=None, choices=[0, 1, 2],
                     help="coloc: time one co-located layout's batch alone (0 MHA 32/32, 1 GQA 32/8, 2 GQA 40/8)")
@@ -541,58 +645,9 @@ def main():
 
     wl = WORKLOADS[args.workload](args, K, W, DevicePool, DeviceSteps)
     stream = torch.cuda.current_stream()
-    launches_per_step = 0
-    cascade = None
-    if hasattr(wl, "prefix_plan") and not args.no_cascade and not args.separate_append:
-        cascade = wl.prefix_plan()
-        for _, buf in wl.tables():
-            buf.use_cascade()
-
-    fuse_sync = cascade is None and not args.separate_append and not args.separate_sync
-    # co-located batches without host tables (the same step repeated): one call
-    multi = (cascade is None and not args.separate_append and not args.separate_batches
-             and len(wl.tables()) > 1 and all(tab is None for tab, _ in wl.tables()))
-
-    def sync_kernels():
-        return sum(tab.counters()["sync_launches"] for tab, _ in wl.tables() if tab is not None)
-
-    def step(ev_pair=None):
-        """host bookkeeping, table sync, then append + attention per batch"""
-        nonlocal launches_per_step
-        nbytes = wl.host_step()
-        n = 0
-        if not fuse_sync:
-            for tab, buf in wl.tables():
-                if tab is not None:
-                    tab.sync(buf.table, buf.lens, stream)
-                    n += 1
-        if ev_pair is not None:
-            ev_pair[0].record(stream)
-        if multi:
-            # every batch's decode kernel as one chain, then the combines
-            K.paged_decode_attn_multi(wl.pool.handle, [buf.batch() for _, buf in wl.tables()], stream)
-            n += 2 * len(wl.tables())
-        for tab, buf in (() if multi else wl.tables()):
-            if fuse_sync and tab is not None:
-                # table sync, append and attention: the decode launch carries
-                # the sync when it fits (else a sync kernel runs first; those
-                # launches are counted from the tables' counters)
-                buf.sync_append_attend(tab, stream)
-                n += 2
-            elif cascade is not None:
-                buf.cascade(cascade, stream=stream)  # plan, attention (fused append), prefix kernel, combine
-                n += 4
-            elif args.separate_append:
-                buf.append(stream)
-                buf.attend(stream)
-                n += 3
-            else:
-                buf.append_attend(stream)  # the append fused into the attention pass
-                n += 2
-        if ev_pair is not None:
-            ev_pair[1].record(stream)
-        launches_per_step = n
-        return nbytes
+    runner = StepRunner(wl, args, K, stream)
+    cascade, fuse_sync, multi = runner.cascade, runner.fuse_sync, runner.multi
+    step, sync_kernels = runner.step, runner.sync_kernels
 
     # No garbage-collector pass inside the timed regions: a full pass over the
     # interpreter's objects (torch's included) stalled the submitting thread
@@ -700,6 +755,14 @@ def main():
     tokens_per_s = tot["tokens"] / (ms * 1e-3)
     e2e_gbs = tot["e2e"] / (e2e_ms * 1e-3) / 1e9
 
+    secondary = None
+    if world == 1 and not args.no_secondary and args.workload == "llama8b":
+        # the other workloads' steps, so that one run records all of them
+        del bufs, pinned
+        secondary = {}
+        for name in ("chains", "coloc", "longctx"):
+            secondary[name] = measure_secondary(name, args, K, W, DevicePool, DeviceSteps, stream, peak)
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and args.workload == "llama8b":
         b = wl.b
@@ -739,20 +802,22 @@ def main():
         "roofline": {"bound": "hbm", "achieved": attn_gbs, "peak": peak, "unit": "GB/s",
                      "frac": attn_gbs / peak, "traffic": traffic,
                      "kernel": step_kernels,
-                     "peak_kind": peak_kind, "call_ms": call_ms, "timed_launches": launches_per_step * args.steps
+                     "peak_kind": peak_kind, "call_ms": call_ms, "timed_launches": runner.launches_per_step * args.steps
                      + extra_sync_launches,
                      "timing": "CUDA events at the ends of the timed region, whose launches are all the "
                                "attention call's kernels: region time / steps",
                      "isolated_call_ms": iso_ms, "isolated_frac": iso_gbs / peak},
         "step_frac_of_peak": gbs / world / peak,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": launches_per_step * args.steps + extra_sync_launches,
+        "gpu_launches": runner.launches_per_step * args.steps + extra_sync_launches,
         "host_us_per_step": host_us,
         "host_cores": pinned_cores,
         "clocks": clk,
         "device_error": err,
         "cpu_baseline": cpu,
     }
+    if secondary is not None:
+        line["secondary_workloads"] = secondary
     if tot["logical"] != tot["dram"]:
         line["logical_gbs"] = tot["logical"] / (ms * 1e-3) / 1e9
     if rank == 0:
