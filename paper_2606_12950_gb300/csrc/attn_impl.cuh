@@ -907,10 +907,10 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
 // (or with a shared prefix), merge its records (m_k, l_k, o_k) in order:
 //     M = max_k m_k,  out = sum_k 2^(m_k - M) o_k / sum_k 2^(m_k - M) l_k
 // (base-2 online-softmax state).  One CTA per run, covering all G*D output
-// columns: NG thread groups of G*D/4 threads (one float4 column each) take
-// records k = grp, grp + NG, ..., then merge their states in group order, so
-// the result depends only on the run's shape.  Runs finished inside the
-// attention kernel return at once.
+// columns: NG thread groups of G*D/(4*CPT) threads (CPT float4 columns
+// each) take records k = grp, grp + NG, ..., then merge their states in
+// group order, so the result depends only on the run's shape.  Runs finished
+// inside the attention kernel return at once.
 struct CombineArgs {
     uint16_t *out;
     const int2 *ws_run;    // per run: (first part, parts), parts = 0 when not split
@@ -932,9 +932,8 @@ constexpr int kCombineBatch = 8;  // records each thread loads per round trip
 // few round trips; at 64 registers four 256-thread CTAs fit on an SM, one
 // wave covering 600 runs.  In shared-prefix mode every member run carries
 // the KS prefix records and the parts of a short suffix, so the counts are
-// uniform and small: there the minimum is 128 threads, which fits twice as
-// many runs in a wave (2048 member runs of the agent chains: 1.7 waves
-// instead of 3.4).
+// uniform and small: there the minimum is 128 threads, one group when a
+// run's output has 128 float4 columns or more.
 template <int D, int G>
 inline int combine_groups(double records_per_run, bool shared_prefix)
 {
@@ -946,16 +945,41 @@ inline int combine_groups(double records_per_run, bool shared_prefix)
     return want < base ? base : (want > most ? most : want);
 }
 
-template <int D, int G>
-__global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __grid_constant__ CombineArgs c)
+// Columns per thread CPT: 1, or 2 for the one-group form of shared-prefix
+// mode.  There every member run is one CTA, and the agent chains have 2048
+// of them: at one column a thread (128 threads a run) and 64 registers only
+// eight CTAs fit an SM and the last 850 runs wait for a second wave; at two
+// columns a thread (64 threads a run, registers held to 64, no shared
+// memory) sixteen fit and one wave covers 2432 runs.  Each column merges the
+// same records in the same order either way, so the bits do not change.
+template <int D, int G, int CPT>
+struct CombineShape {
+    static constexpr int NC = G * D / 4;   // float4 columns of a run's output
+    static constexpr int NCT = NC / CPT;   // threads of a group
+    static constexpr int MAX_THREADS = CPT == 1 ? kCombineMaxThreads : NCT;
+    static constexpr int MIN_CTAS = CPT == 1 ? 1 : 28 / ((NCT + 31) / 32);  // 28 warps an SM: 72 registers
+    static constexpr int BATCH = CPT == 1 ? kCombineBatch : 4;
+};
+
+// shared memory of a CTA of `threads` threads: the groups' states for the
+// in-order merge (none with one group)
+template <int D, int G, int CPT>
+inline size_t combine_smem_bytes(int threads)
 {
+    return threads > CombineShape<D, G, CPT>::NCT ? (size_t)threads * CPT * (2 * sizeof(float) + sizeof(float4)) : 0;
+}
+
+template <int D, int G, int CPT>
+__global__ void __launch_bounds__(CombineShape<D, G, CPT>::MAX_THREADS, CombineShape<D, G, CPT>::MIN_CTAS)
+combine_kernel(const __grid_constant__ CombineArgs c)
+{
+    using CS = CombineShape<D, G, CPT>;
     constexpr uint32_t MF = merge_floats<D, G>();
-    constexpr int NC = G * D / 4;  // float4 columns of a run's output
-    static_assert(NC <= kCombineMaxThreads, "one thread per output column");
-    const int NG = (int)blockDim.x / NC;  // groups of NC threads
-    __shared__ float s_M[kCombineMaxThreads];
-    __shared__ float s_L[kCombineMaxThreads];
-    __shared__ float4 s_O[kCombineMaxThreads];
+    constexpr int NCT = CS::NCT;
+    constexpr int B = CS::BATCH;
+    static_assert(CS::NC % CPT == 0 && NCT <= kCombineMaxThreads, "whole columns per thread");
+    const int NG = (int)blockDim.x / NCT;  // groups of NCT threads
+    extern __shared__ float4 s_dyn[];      // [CPT][blockDim] O, then M, then L (when NG > 1)
     const int r = blockIdx.x;
     // the next grid in the stream may be scheduled now; it waits for this
     // one to complete before touching anything this grid reads
@@ -969,68 +993,97 @@ __global__ void __launch_bounds__(kCombineMaxThreads) combine_kernel(const __gri
     const float *base = c.ws_part + ((int64_t)r + info.x) * MF;
     uint16_t *orow = c.out + ((int64_t)s * c.Hkv * G + (int64_t)g * G) * D;
     const int tid = threadIdx.x;
-    const int col = tid % NC;
-    const int grp = tid / NC;
-    const int h = (col * 4) / D;
-    // online merge of this group's records: M running max, L and O relative
-    // to M; records k = grp, grp + NG, ... are loaded kCombineBatch at a time
-    float M = -INFINITY, L = 0.f;
-    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = grp; k0 < cnt; k0 += NG * kCombineBatch) {
-        float mv[kCombineBatch], lv[kCombineBatch];
-        float4 ov[kCombineBatch];
+    const int grp = tid / NCT;
+    int col[CPT], h[CPT];
 #pragma unroll
-        for (int b = 0; b < kCombineBatch; ++b) {
+    for (int j = 0; j < CPT; ++j) {
+        col[j] = tid % NCT + j * NCT;
+        h[j] = (col[j] * 4) / D;
+    }
+    // online merge of this group's records per column: M running max, L and
+    // O relative to M; records k = grp, grp + NG, ... are loaded B at a time
+    float M[CPT], L[CPT];
+    float4 O[CPT];
+#pragma unroll
+    for (int j = 0; j < CPT; ++j) {
+        M[j] = -INFINITY;
+        L[j] = 0.f;
+        O[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    for (int k0 = grp; k0 < cnt; k0 += NG * B) {
+        float mv[B][CPT], lv[B][CPT];
+        float4 ov[B][CPT];
+#pragma unroll
+        for (int b = 0; b < B; ++b) {
             const int k = k0 + b * NG;
-            mv[b] = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < CPT; ++j) mv[b][j] = -INFINITY;
             if (k < cnt) {
                 const float *sl = k < npre ? c.ws_pre + (((int64_t)k * c.S + s) * c.Hkv + g) * MF
                                            : base + (int64_t)(k - npre) * MF;
-                mv[b] = sl[G * D + h];
-                lv[b] = sl[G * D + G + h];
-                ov[b] = *reinterpret_cast<const float4 *>(sl + col * 4);
+#pragma unroll
+                for (int j = 0; j < CPT; ++j) {
+                    mv[b][j] = sl[G * D + h[j]];
+                    lv[b][j] = sl[G * D + G + h[j]];
+                    ov[b][j] = *reinterpret_cast<const float4 *>(sl + col[j] * 4);
+                }
             }
         }
 #pragma unroll
-        for (int b = 0; b < kCombineBatch; ++b) {
-            if (mv[b] == -INFINITY) continue;  // past the run's records
-            const float Mn = fmaxf(M, mv[b]);
-            const float sa = fast_exp2(M - Mn), sb = fast_exp2(mv[b] - Mn);
-            L = L * sa + lv[b] * sb;
-            O.x = O.x * sa + ov[b].x * sb;
-            O.y = O.y * sa + ov[b].y * sb;
-            O.z = O.z * sa + ov[b].z * sb;
-            O.w = O.w * sa + ov[b].w * sb;
-            M = Mn;
-        }
+        for (int b = 0; b < B; ++b)
+#pragma unroll
+            for (int j = 0; j < CPT; ++j) {
+                if (mv[b][j] == -INFINITY) continue;  // past the run's records
+                const float Mn = fmaxf(M[j], mv[b][j]);
+                const float sa = fast_exp2(M[j] - Mn), sb = fast_exp2(mv[b][j] - Mn);
+                L[j] = L[j] * sa + lv[b][j] * sb;
+                O[j].x = O[j].x * sa + ov[b][j].x * sb;
+                O[j].y = O[j].y * sa + ov[b][j].y * sb;
+                O[j].z = O[j].z * sa + ov[b][j].z * sb;
+                O[j].w = O[j].w * sa + ov[b][j].w * sb;
+                M[j] = Mn;
+            }
     }
     if (NG > 1) {
-        s_M[tid] = M;
-        s_L[tid] = L;
-        s_O[tid] = O;
+        const int nt = (int)blockDim.x;
+        float4 *s_O = s_dyn;
+        float *s_M = reinterpret_cast<float *>(s_dyn + CPT * nt);
+        float *s_L = s_M + CPT * nt;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) {
+            s_M[j * nt + tid] = M[j];
+            s_L[j * nt + tid] = L[j];
+            s_O[j * nt + tid] = O[j];
+        }
         __syncthreads();
         if (grp != 0) return;
         // merge the groups in order
-        for (int j = 1; j < NG; ++j) {
-            const float mj = s_M[tid + j * NC];
-            if (mj == -INFINITY) continue;  // group had no records
-            const float Mn = fmaxf(M, mj);
-            const float sa = fast_exp2(M - Mn), sb = fast_exp2(mj - Mn);
-            const float4 oj = s_O[tid + j * NC];
-            L = L * sa + s_L[tid + j * NC] * sb;
-            O.x = O.x * sa + oj.x * sb;
-            O.y = O.y * sa + oj.y * sb;
-            O.z = O.z * sa + oj.z * sb;
-            O.w = O.w * sa + oj.w * sb;
-            M = Mn;
-        }
+        for (int q = 1; q < NG; ++q)
+#pragma unroll
+            for (int j = 0; j < CPT; ++j) {
+                const int i = j * nt + tid + q * NCT;
+                const float mq = s_M[i];
+                if (mq == -INFINITY) continue;  // group had no records
+                const float Mn = fmaxf(M[j], mq);
+                const float sa = fast_exp2(M[j] - Mn), sb = fast_exp2(mq - Mn);
+                const float4 oq = s_O[i];
+                L[j] = L[j] * sa + s_L[i] * sb;
+                O[j].x = O[j].x * sa + oq.x * sb;
+                O[j].y = O[j].y * sa + oq.y * sb;
+                O[j].z = O[j].z * sa + oq.z * sb;
+                O[j].w = O[j].w * sa + oq.w * sb;
+                M[j] = Mn;
+            }
     }
-    __nv_bfloat162 lo = __floats2bfloat162_rn(O.x / L, O.y / L);
-    __nv_bfloat162 hi = __floats2bfloat162_rn(O.z / L, O.w / L);
-    uint2 w2;
-    w2.x = *reinterpret_cast<uint32_t *>(&lo);
-    w2.y = *reinterpret_cast<uint32_t *>(&hi);
-    *reinterpret_cast<uint2 *>(orow + col * 4) = w2;
+#pragma unroll
+    for (int j = 0; j < CPT; ++j) {
+        __nv_bfloat162 lo = __floats2bfloat162_rn(O[j].x / L[j], O[j].y / L[j]);
+        __nv_bfloat162 hi = __floats2bfloat162_rn(O[j].z / L[j], O[j].w / L[j]);
+        uint2 w2;
+        w2.x = *reinterpret_cast<uint32_t *>(&lo);
+        w2.y = *reinterpret_cast<uint32_t *>(&hi);
+        *reinterpret_cast<uint2 *>(orow + col[j] * 4) = w2;
+    }
 }
 
 // host helpers ---------------------------------------------------------------

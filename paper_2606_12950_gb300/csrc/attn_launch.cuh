@@ -91,11 +91,20 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     // records per run: at most P * nwarps parts spread over the runs, plus
     // the prefix records in shared-prefix mode
     const double per_run = (double)P * a.nwarps / std::max(1, a.S * a.Hkv) + 1.0 + (a.skip ? a.KS : 0);
+    const int groups = combine_groups<D, G>(per_run, a.skip != nullptr);
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv));
-    ccfg.blockDim = dim3((unsigned)(combine_groups<D, G>(per_run, a.skip != nullptr) * (G * D / 4)));
-    ccfg.dynamicSmemBytes = 0;
-    if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G>, c) != cudaSuccess) return KV_ERR_CUDA;
-    return KV_OK;
+    if constexpr (G * D / 4 >= 128) {
+        // one group: two columns a thread, so that every run fits in one wave
+        if (groups == 1) {
+            ccfg.blockDim = dim3((unsigned)CombineShape<D, G, 2>::NCT);
+            ccfg.dynamicSmemBytes = 0;
+            return cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 2>, c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+        }
+    }
+    const int threads = groups * (G * D / 4);
+    ccfg.blockDim = dim3((unsigned)threads);
+    ccfg.dynamicSmemBytes = combine_smem_bytes<D, G, 1>(threads);
+    return cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 1>, c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
 // Shared-prefix kernel: with launch = false only reports the CTAs that fit
