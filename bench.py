@@ -501,6 +501,8 @@ class StepRunner:
             for _, buf in wl.tables():
                 buf.use_cascade()
         self.fuse_sync = self.cascade is None and not args.separate_append and not args.separate_sync
+        # shared prefix: the table sync rides in the kernel that writes the plan
+        self.cascade_sync = self.cascade is not None and not args.separate_sync
         # co-located batches without host tables (the same step repeated): one call
         self.multi = (self.cascade is None and not args.separate_append and not args.separate_batches
                       and len(wl.tables()) > 1 and all(tab is None for tab, _ in wl.tables()))
@@ -514,7 +516,7 @@ class StepRunner:
         wl, args, K, stream = self.wl, self.args, self.K, self.stream
         nbytes = wl.host_step()
         n = 0
-        if not self.fuse_sync:
+        if not self.fuse_sync and not self.cascade_sync:
             for tab, buf in wl.tables():
                 if tab is not None:
                     tab.sync(buf.table, buf.lens, stream)
@@ -533,7 +535,12 @@ class StepRunner:
                 buf.sync_append_attend(tab, stream)
                 n += 2
             elif self.cascade is not None:
-                buf.cascade(self.cascade, stream=stream)  # plan, attention (fused append), prefix kernel, combine
+                # plan (with the table sync when it fits), prefix kernel,
+                # attention with the fused append, combine
+                if self.cascade_sync:
+                    buf.sync_cascade(tab, self.cascade, stream=stream)
+                else:
+                    buf.cascade(self.cascade, stream=stream)
                 n += 4
             elif args.separate_append:
                 buf.append(stream)
@@ -608,7 +615,7 @@ def main():
     ap.add_argument("--separate-batches", action="store_true",
                     help="one call per co-located batch instead of one paged_decode_attn_multi call")
     ap.add_argument("--separate-sync", action="store_true",
-                    help="table sync with its own kernel instead of carried by the decode launch")
+                    help="table sync with its own kernel instead of carried by the decode (or plan) launch")
     ap.add_argument("--pool", default="fixed", choices=["fixed", "vmm"],
                     help="llama8b: a fixed device buffer, or the VMM-backed elastic pool")
     ap.add_argument("--no-cascade", action="store_true",
@@ -647,6 +654,7 @@ def main():
     stream = torch.cuda.current_stream()
     runner = StepRunner(wl, args, K, stream)
     cascade, fuse_sync, multi = runner.cascade, runner.fuse_sync, runner.multi
+    cascade_sync = runner.cascade_sync
     step, sync_kernels = runner.step, runner.sync_kernels
 
     # No garbage-collector pass inside the timed regions: a full pass over the
@@ -678,7 +686,8 @@ def main():
         step_bytes.append(step())
     t_end.record(stream)
     host_us = (time.perf_counter() - h0) * 1e6 / args.steps  # host submission time per step
-    extra_sync_launches = sync_kernels() - sync0 if fuse_sync else 0
+    # sync kernels the calls launched themselves (syncs too large to carry)
+    extra_sync_launches = sync_kernels() - sync0 if fuse_sync or cascade_sync else 0
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = t_start.elapsed_time(t_end)
@@ -789,7 +798,8 @@ def main():
     config = {"workload": wl.name, **wl.config, "num_splits": args.num_splits, "variant": args.variant,
               "pool": args.pool if args.workload == "llama8b" else "fixed",
               "append": "separate kernel" if args.separate_append else "fused into attention",
-              "table_sync": ("carried by the decode launch when it fits" if fuse_sync else "separate kernel"),
+              "table_sync": ("carried by the decode launch when it fits" if fuse_sync else
+                             "carried by the plan launch when it fits" if cascade_sync else "separate kernel"),
               "batches": "one paged_decode_attn_multi call" if multi else "one call per batch",
               "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
                                 else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,

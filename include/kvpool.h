@@ -624,6 +624,27 @@ int paged_decode_attn_cascade(kv_pool *pool, int layout, const uint16_t *q, cons
                               size_t ws_bytes, void *stream);
 
 /*
+ * kv_seqtab_sync(t, dev_table, dev_ctx_lens, stream) followed by
+ * paged_decode_attn_cascade over the table's first S rows (layout and
+ * max_blocks taken from the table), with the sync carried by the cascade
+ * call's first launch: when the plan's words, the table's S lengths and
+ * two words per entry changed since the last sync make at most 4080 words,
+ * the kernel that writes the plan to the workspace also writes the lengths
+ * and the changed entries to dev_ctx_lens / dev_table (the separate sync
+ * kernel and its hand-off drop out of the step).  Otherwise (the first
+ * sync, or more changes than fit) the call runs kv_seqtab_sync first.
+ * n_groups = 0 is paged_decode_attn_seqtab with num_splits = 0; S = 0 is
+ * kv_seqtab_sync alone.  Results, device table and lengths afterwards are
+ * those of the two calls; errors are theirs (KV_ERR_INVALID_ARG also when t
+ * is not over `pool` or S > max_seqs).
+ */
+int paged_decode_attn_cascade_seqtab(kv_pool *pool, kv_seqtab *t, const uint16_t *q, const uint16_t *k_new,
+                                     const uint16_t *v_new, uint16_t *out, int32_t *dev_table,
+                                     int32_t *dev_ctx_lens, int S, int Hq, float scale,
+                                     const kv_prefix_group *groups, int n_groups, const int32_t *members,
+                                     void *workspace, size_t ws_bytes, void *stream);
+
+/*
  * paged_decode_attn for callers that cannot allocate device memory.  The
  * paper has no counterpart; this is a service of this library.  Callers that
  * cannot hand over a workspace include a server whose KV pool already holds

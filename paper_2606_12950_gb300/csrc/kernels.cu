@@ -130,36 +130,64 @@ int dispatch(int variant, int D, int G, const CUtensorMap *tmap, const kvp::Attn
     return kvp_attn_d128(variant, G, tmap, a, P_req, sms, st, what, P_out);
 }
 
+// a host sequence table whose pending changes travel with a launch (the
+// decode launch, or the plan kernel's in shared-prefix mode)
+struct FusedSync {
+    kv_seqtab *t;
+    int32_t *dev_table;
+    int32_t *dev_lens;
+};
+
 // The shared-prefix plan, carried as this kernel's parameters, into the
 // workspace: the whole plan for the prefix kernel, and the per-sequence
 // skips (its last S words) where the decode kernel (suffix tiles start
-// there) and the combine read them.  It waits for the previous grid first:
-// the previous step's kernels may still read the old plan and skips.  The
-// parameter block comes in two sizes so that a small plan does not pay for
-// copying the largest one into every launch (host and device time).
+// there) and the combine read them; with a fused table sync also a
+// sequence table's lengths and changed entries, into the device lengths
+// and table (what the sync kernel would write), which saves that kernel's
+// launch and its grid-to-grid hand-off.  It waits for the previous grid
+// first: the previous step's kernels may still read the old plan, skips,
+// lengths and table.  The parameter block comes in three sizes so that a
+// small plan does not pay for copying the largest one into every launch
+// (host and device time).
 template <int W>
 struct PlanParams {
     int32_t *ws_plan;
     int32_t *ws_skip;
-    int32_t n_words;
+    int32_t *sync_table;  // fused table sync: null for none
+    int32_t *sync_lens;
+    int32_t n_words;      // plan words
     int32_t S;
-    int32_t words[W];
+    int32_t sync_nlens;
+    int32_t sync_npatch;
+    int32_t words[W];  // the plan, then sync_nlens lengths, then sync_npatch (flat index, value) pairs
 };
 
 template <int W>
 __global__ void cascade_plan_kernel(const __grid_constant__ PlanParams<W> p)
 {
+    // the grids before (the previous step's kernels, which read the plan,
+    // the lengths and the table) have completed after this wait; the grid
+    // after waits for this one to complete before it reads any of them
     kvp::grid_dependency_wait();
     kvp::grid_launch_dependents();
     for (int i = threadIdx.x; i < p.n_words; i += blockDim.x) p.ws_plan[i] = p.words[i];
     const int32_t *skip = p.words + (p.n_words - p.S);
     for (int s = threadIdx.x; s < p.S; s += blockDim.x) p.ws_skip[s] = skip[s];
+    if (p.sync_table) {
+        const int32_t *lw = p.words + p.n_words, *pw = lw + p.sync_nlens;
+        for (int i = threadIdx.x; i < p.sync_nlens; i += blockDim.x) p.sync_lens[i] = lw[i];
+        for (int j = threadIdx.x; j < p.sync_npatch; j += blockDim.x) p.sync_table[pw[2 * j]] = pw[2 * j + 1];
+    }
 }
 
+// parameter blocks of three sizes (a launch's host cost grows with its
+// parameter bytes): about 4, 8 and 16 KB
 constexpr int kPlanSmallWords = 1024;
+constexpr int kPlanMidWords = 2040;
 
 template <int W>
-int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip, cudaStream_t st)
+int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip,
+                        const FusedSync *sync, cudaStream_t st)
 {
     static thread_local std::unique_ptr<PlanParams<W>> buf(new PlanParams<W>());
     PlanParams<W> *p = buf.get();
@@ -168,6 +196,25 @@ int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_pl
     p->n_words = n_words;
     p->S = S;
     std::copy(words, words + n_words, p->words);
+    p->sync_table = nullptr;
+    p->sync_lens = nullptr;
+    p->sync_nlens = 0;
+    p->sync_npatch = 0;
+    if (sync) {
+        const kv_seqtab *t = sync->t;
+        const int nl = t->S, np = (int)t->changed.size();
+        int32_t *w = p->words + n_words;
+        for (int i = 0; i < nl; ++i) w[i] = t->lens[(size_t)i];
+        for (int j = 0; j < np; ++j) {
+            const int32_t idx = t->changed[(size_t)j];
+            w[nl + 2 * j] = idx;
+            w[nl + 2 * j + 1] = t->table[(size_t)idx];
+        }
+        p->sync_table = sync->dev_table;
+        p->sync_lens = sync->dev_lens;
+        p->sync_nlens = nl;
+        p->sync_npatch = np;
+    }
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -180,11 +227,23 @@ int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_pl
     return cudaLaunchKernelEx(&cfg, cascade_plan_kernel<W>, *p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
-int cascade_plan_run(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip, cudaStream_t st)
+// words the plan kernel carries: the plan's, plus the sync's lengths and
+// changed entries when it is fused
+inline size_t plan_sync_words(int n_words, const FusedSync *sync)
 {
-    if (n_words <= kPlanSmallWords)
-        return cascade_plan_launch<kPlanSmallWords>(words, n_words, S, ws_plan, ws_skip, st);
-    return cascade_plan_launch<kvp::kCascadeWords>(words, n_words, S, ws_plan, ws_skip, st);
+    return (size_t)n_words + (sync ? (size_t)sync->t->S + 2 * sync->t->changed.size() : 0);
+}
+
+int cascade_plan_run(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip,
+                     const FusedSync *sync, cudaStream_t st)
+{
+    const size_t n = plan_sync_words(n_words, sync);
+    if (n <= (size_t)kPlanSmallWords)
+        return cascade_plan_launch<kPlanSmallWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
+    if (n <= (size_t)kPlanMidWords)
+        return cascade_plan_launch<kPlanMidWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
+    if (n > (size_t)kvp::kCascadeWords) return KV_ERR_INVALID_ARG;  // the caller syncs separately first
+    return cascade_plan_launch<kvp::kCascadeWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
 }
 
 // workspace: per-run (first part, parts) as int2 (padded to 256 bytes),
@@ -285,13 +344,6 @@ struct CascadePlan {
     const kv_prefix_group *groups;
     int n_groups;
     const int32_t *members;
-};
-
-// a host sequence table whose pending changes travel with the decode launch
-struct FusedSync {
-    kv_seqtab *t;
-    int32_t *dev_table;
-    int32_t *dev_lens;
 };
 
 int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
@@ -456,9 +508,22 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.KS = c->KS;
     rc = ensure_tmap(p, layout);
     if (rc) return rc;
+    // a table sync that does not fit the plan kernel's parameters (or a
+    // table never written to the device) runs as its own launches first
+    if (sync && (sync->t->full_dirty || plan_sync_words(n_words, sync) > (size_t)kvp::kCascadeWords)) {
+        rc = kv_seqtab_sync(sync->t, sync->dev_table, sync->dev_lens, stream);
+        if (rc) return rc;
+        sync = nullptr;
+    }
     rc = cascade_plan_run(words_buf.data(), n_words, S, reinterpret_cast<int32_t *>(ws + plan_off), c->ws_skip,
-                          (cudaStream_t)stream);
+                          sync, (cudaStream_t)stream);
     if (rc) return rc;
+    if (sync) {
+        kv_seqtab *t = sync->t;
+        t->counters.entries_uploaded += (int64_t)t->changed.size();
+        for (int32_t idx : t->changed) t->pending[(size_t)idx] = 0;
+        t->changed.clear();
+    }
     rc = cascade_dispatch(L.head_dim, G, &p->tmap[layout], c, pre_ctas, p->sm_count, (cudaStream_t)stream, true,
                           &P_pre);
     if (rc) return rc;
@@ -622,4 +687,22 @@ extern "C" int paged_decode_attn_cascade(kv_pool *p, int layout, const uint16_t 
     const CascadePlan plan{groups, n_groups, members};
     return attn_call(p, layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, max_blocks, S, Hq, scale, 0,
                      workspace, ws_bytes, stream, &plan);
+}
+
+extern "C" int paged_decode_attn_cascade_seqtab(kv_pool *p, kv_seqtab *t, const uint16_t *q, const uint16_t *k_new,
+                                                const uint16_t *v_new, uint16_t *out, int32_t *dev_table,
+                                                int32_t *dev_ctx_lens, int S, int Hq, float scale,
+                                                const kv_prefix_group *groups, int n_groups, const int32_t *members,
+                                                void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!p || !t || t->pool != p || !dev_table || !dev_ctx_lens || S < 0 || S > t->S) return KV_ERR_INVALID_ARG;
+    if (n_groups < 0 || (!k_new) != (!v_new)) return KV_ERR_INVALID_ARG;
+    if (n_groups == 0)
+        return paged_decode_attn_seqtab(p, t, q, k_new, v_new, out, dev_table, dev_ctx_lens, S, Hq, scale, 0,
+                                        workspace, ws_bytes, stream);
+    if (S == 0) return kv_seqtab_sync(t, dev_table, dev_ctx_lens, stream);
+    const CascadePlan plan{groups, n_groups, members};
+    const FusedSync sync{t, dev_table, dev_ctx_lens};
+    return attn_call(p, t->layout, q, k_new, v_new, out, dev_table, dev_ctx_lens, t->max_blocks, S, Hq, scale, 0,
+                     workspace, ws_bytes, stream, &plan, &sync);
 }

@@ -188,6 +188,7 @@ def lib() -> ctypes.CDLL:
             "kv_budget_destroy": [P],
             "kv_budget_used": [P, ctypes.POINTER(U64)],
             "paged_decode_attn_cascade": [P, I, P, P, P, P, P, P, I, I, I, F, P, I, P, P, SZ, P],
+            "paged_decode_attn_cascade_seqtab": [P, P, P, P, P, P, P, P, I, I, F, P, I, P, P, SZ, P],
             "kv_seqtab_create": [P, I, I, I, ctypes.POINTER(P)],
             "kv_seqtab_destroy": [P],
             "kv_seq_reserve": [P, I, I64],
@@ -503,6 +504,20 @@ def paged_decode_attn_cascade(pool, layout: int, q, k_new, v_new, out, dev_table
                                            float(scale), ctypes.addressof(plan.groups), plan.n_groups,
                                            ctypes.addressof(plan.members), _addr(workspace), int(ws_bytes),
                                            _stream(stream)))
+
+
+def paged_decode_attn_cascade_seqtab(pool, seqtab, q, k_new, v_new, out, dev_table, dev_ctx_lens, S: int,
+                                     Hq: int, scale: float, plan: PrefixPlan, workspace, ws_bytes: int,
+                                     stream=None) -> None:
+    """kv_seqtab_sync + paged_decode_attn_cascade, the sync carried by the
+    kernel that writes the plan when it fits there."""
+    h = seqtab.handle if isinstance(seqtab, SeqTab) else seqtab
+    _check("paged_decode_attn_cascade_seqtab",
+           lib().paged_decode_attn_cascade_seqtab(pool, h, _addr(q), _addr(k_new), _addr(v_new), _addr(out),
+                                                  _addr(dev_table), _addr(dev_ctx_lens), int(S), int(Hq),
+                                                  float(scale), ctypes.addressof(plan.groups), plan.n_groups,
+                                                  ctypes.addressof(plan.members), _addr(workspace), int(ws_bytes),
+                                                  _stream(stream)))
 
 
 def kv_set_attn_variant(pool, variant: int) -> None:

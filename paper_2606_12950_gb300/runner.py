@@ -300,3 +300,10 @@ class DeviceSteps:
                                     self.v_new if fused else None, self.out, self.table, self.lens,
                                     self.max_blocks, self.S, self.Hq, self.scale, plan, self.ws,
                                     self.ws.numel(), stream)
+
+    def sync_cascade(self, seqtab, plan, stream=None) -> None:
+        """seqtab's table sync, then shared-prefix attention with the fused
+        append; the sync rides in the kernel that writes the plan when it fits."""
+        K.paged_decode_attn_cascade_seqtab(self.pool.handle, seqtab, self.q, self.k_new, self.v_new, self.out,
+                                           self.table, self.lens, self.S, self.Hq, self.scale, plan, self.ws,
+                                           self.ws.numel(), stream)

@@ -6,8 +6,9 @@ not the CUDA path); the oracle mirrors every append on its own copy of the
 pool.  Every sequence's output is compared with the oracle on every checked
 step (the oracle spread over the host cores, ``par_oracle``), the pool
 bit-exactly.  The full-size tests drive the entry points and launch
-configuration the benchmark times for each workload: the table sync and the
-cascade call with the fused append (agent chains), one
+configuration the benchmark times for each workload: the cascade call with
+the fused append and the table sync carried by its plan kernel (agent
+chains), one
 paged_decode_attn_multi call (co-location), paged_decode_attn_seqtab with
 the fused sync and append (long context).
 """
@@ -49,12 +50,15 @@ def _check_all(got, host_pool, n_pages, page_elems, bs, Hkv, d, q, table, lens, 
 
 
 def _run_chains(n_chains, steps, median, max_out, seed=1003, check_every=1, cascade=False,
-                until_stage_end=False):
+                until_stage_end=False, sync_in_call=False, bits=None):
     """Agent chains driven as the benchmark drives them: the sequence table's
-    sync, then the cascade call with the fused append (shared-prefix mode)
-    or the append and attention calls.  Every chain is checked on every
-    checked step.  With until_stage_end the run goes on (up to ``steps``)
-    until two steps after the first stage boundary."""
+    sync, then the cascade call with the fused append (shared-prefix mode;
+    with sync_in_call one paged_decode_attn_cascade_seqtab call, the sync
+    carried by its plan kernel) or the append and attention calls.  Every
+    chain is checked on every checked step.  With until_stage_end the run
+    goes on (up to ``steps``) until two steps after the first stage
+    boundary.  ``bits``, a list, receives every step's output bits, device
+    lengths and table, and the run's sync-kernel launches after each step."""
     from paper_2606_12950_gb300.runner import DevicePool, DeviceSteps
     from paper_2606_12950_gb300.schedules import AgentChains
 
@@ -78,14 +82,20 @@ def _run_chains(n_chains, steps, median, max_out, seed=1003, check_every=1, casc
         ch.step()
         q, kn, vn = W.step_rows(seed, step, n_chains, Hq, Hkv, d)
         buf.inputs.copy_(_dev_bits(np.concatenate([q.reshape(-1), kn.reshape(-1), vn.reshape(-1)])))
-        buf.sync(ch.tab)
-        if cascade:
+        if cascade and sync_in_call:
+            buf.sync_cascade(ch.tab, plan)
+        elif cascade:
+            buf.sync(ch.tab)
             buf.cascade(plan)
         else:
+            buf.sync(ch.tab)
             buf.append()
             buf.attend()
         torch.cuda.synchronize()
         got = buf.out.float().cpu().numpy().astype(np.float64)
+        if bits is not None:
+            bits.append((buf.out.view(torch.int16).cpu().numpy().copy(), buf.lens.cpu().numpy().copy(),
+                         buf.table.cpu().numpy().copy(), ch.tab.counters()["sync_launches"]))
         table, lens = ch.tab.host()
         table, lens = table[:n_chains], lens[:n_chains]
         oracle.append(host_pool, n_pages, page_elems, bs, Hkv, d, kn, vn, table, lens, inplace=True)
@@ -114,15 +124,37 @@ def test_agent_chains_full_size():
 
 def test_agent_chains_full_size_cascade_across_a_stage_boundary():
     """The same 256 chains through shared-prefix attention, as the benchmark
-    runs them (table sync, then the cascade call with the fused append): the
+    runs them (one cascade call with the fused append, the table sync
+    carried by its plan kernel): the
     2048-token prompt attended once per KV head for all chains, each chain's
     own context streamed and merged.  The run goes past the first stage
     boundary (a trim and a new stage's reservation; with this seed the
     first stage ends at step 24); every chain is checked on every fourth
     step and on every step from the boundary on."""
     ends, done, misses, boundary, checked = _run_chains(256, steps=64, median=300.0, max_out=4096,
-                                                        check_every=4, cascade=True, until_stage_end=True)
+                                                        check_every=4, cascade=True, until_stage_end=True,
+                                                        sync_in_call=True)
     assert boundary is not None and ends >= 1 and checked >= 8
+
+
+def test_table_sync_carried_by_the_plan_kernel_gives_the_separate_sync_bits():
+    """paged_decode_attn_cascade_seqtab against kv_seqtab_sync followed by
+    paged_decode_attn_cascade, on the same short-stage schedule (stage ends,
+    trims, chain releases, new chains re-sharing the prefix): on every step
+    the same output bits, device lengths and table; the first step (a table
+    never written to the device) takes the separate sync, every later one
+    launches no sync kernel; both runs match the oracle on every fourth
+    step."""
+    fused, separate = [], []
+    _run_chains(48, steps=40, median=5.0, max_out=40, check_every=4, cascade=True, sync_in_call=True,
+                bits=fused)
+    _run_chains(48, steps=40, median=5.0, max_out=40, check_every=4, cascade=True, bits=separate)
+    assert len(fused) == len(separate) == 40
+    for i, (f, r) in enumerate(zip(fused, separate)):
+        for a, b in zip(f[:3], r[:3]):
+            assert np.array_equal(a, b), i
+    assert fused[0][3] >= 1 and fused[-1][3] == fused[0][3]  # no sync kernel after the first step
+    assert separate[-1][3] >= separate[0][3] + 39
 
 
 def test_agent_chains_stage_turnover_cascade():
