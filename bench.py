@@ -495,6 +495,10 @@ class StepRunner:
     def __init__(self, wl, args, K, stream):
         self.wl, self.args, self.K, self.stream = wl, args, K, stream
         self.launches_per_step = 0
+        # a step's decode kernel may start while the previous step's combine
+        # finishes (kv_set_attn_step_overlap)
+        self.step_overlap = not getattr(args, "no_step_overlap", False)
+        wl.pool.set_step_overlap(self.step_overlap)
         self.cascade = None
         if hasattr(wl, "prefix_plan") and not args.no_cascade and not args.separate_append:
             self.cascade = wl.prefix_plan()
@@ -618,6 +622,8 @@ def main():
                     help="table sync with its own kernel instead of carried by the decode (or plan) launch")
     ap.add_argument("--pool", default="fixed", choices=["fixed", "vmm"],
                     help="llama8b: a fixed device buffer, or the VMM-backed elastic pool")
+    ap.add_argument("--no-step-overlap", action="store_true",
+                    help="each step's decode kernel waits for the previous step's combine to complete first")
     ap.add_argument("--no-cascade", action="store_true",
                     help="agent chains: stream the shared prefix per chain instead of once per KV head")
     args = ap.parse_args()
@@ -801,6 +807,7 @@ def main():
               "table_sync": ("carried by the decode launch when it fits" if fuse_sync else
                              "carried by the plan launch when it fits" if cascade_sync else "separate kernel"),
               "batches": "one paged_decode_attn_multi call" if multi else "one call per batch",
+              "step_overlap": runner.step_overlap,
               "shared_prefix": ("attended once per KV head for all sharers (cascade)" if cascade is not None
                                 else "streamed per sequence") if hasattr(wl, "prefix_plan") else None,
               "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}

@@ -683,6 +683,27 @@ int paged_decode_attn_noalloc(kv_pool *pool, int layout, const uint16_t *q, uint
  */
 int kv_set_attn_variant(kv_pool *pool, int variant);
 
+/*
+ * Step overlap for later attention calls on this pool (0 = off, the
+ * default; 1 = on).  On, a paged_decode_attn, paged_decode_attn_append or
+ * paged_decode_attn_seqtab call (and the allocation-free call) whose stream
+ * last received, from this library, the split-K combine of an earlier
+ * attention call starts its decode kernel while that combine is still
+ * finishing: the decode kernel reads the lengths, the table and the pool
+ * and starts streaming at once, and waits for the combine before it writes
+ * the output or the workspace.  That is safe because the combine releases
+ * the next kernel only after everything before it in the stream has
+ * completed.  Any other launch or copy of this library on the stream in
+ * between (a table sync, an append, an upload) turns it off for the next
+ * call, and so does a stream the library has not seen.  Results are the
+ * same bits either way.  The caller's side of the contract: work of
+ * others between two attention calls on one stream must not be launched as
+ * a programmatic dependent that releases its own dependents before it has
+ * finished writing (ordinary kernels and copies are fine), and one host
+ * thread submits to the stream at a time.
+ */
+int kv_set_attn_step_overlap(kv_pool *pool, int on);
+
 /* Library version string (static storage). */
 const char *kv_version(void);
 

@@ -36,7 +36,10 @@
 // Alone it releases the next grid and waits for the one before; as part of
 // a chain (beside the shared-prefix kernel, or the later batches of several
 // co-located ones) it starts without waiting, reads what earlier grids wrote
-// through L2 only, and waits at its end (AttnArgs::chain).  The step's
+// through L2 only, and waits at its end (AttnArgs::chain).  Right after a
+// split-K combine (step overlap) it starts without waiting too, while the
+// combine finishes, and waits before its first write of the output or the
+// workspace, which the combine uses.  The step's
 // table sync may ride in its parameters (AttnArgs::sync_words); a grid
 // alone then computes its work split from those lengths before its wait.
 //
@@ -74,8 +77,9 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
 // Loads of data written by earlier grids: through L2 only (ld.global.cg) when
 // the kernel did not wait for the grid before it (a chained grid: beside the
-// shared-prefix kernel, or a later batch of paged_decode_attn_multi), so that
-// no line an earlier kernel left in this SM's L1 is read; plain otherwise.
+// shared-prefix kernel, a later batch of paged_decode_attn_multi, or a step
+// overlapping the previous step's combine), so that no line an earlier
+// kernel left in this SM's L1 is read; plain otherwise.
 template <class T>
 __device__ __forceinline__ T ld_prior(const T *p, bool l2_only)
 {
@@ -119,7 +123,11 @@ struct AttnArgs {
     // place in a chain of grids: 0 alone (release the next grid, then wait
     // for the one before); 1 first of a chain (wait, then release: the next
     // grid relies on this wait); 2 chained (release, no wait at the start,
-    // a wait at every exit: see the kernel)
+    // a wait at every exit: see the kernel); 3 right after a split-K combine
+    // of this library, which released this grid only after its own wait, so
+    // every grid before that combine has completed (release, no wait at the
+    // start, a wait before the first write of the output or the workspace,
+    // which the combine still uses, and at every exit)
     int32_t chain;
     // fused table sync (paged_decode_attn_seqtab): this step's lengths of
     // rows [0, sync_nlens) and its changed table entries travel here.  The
@@ -518,7 +526,7 @@ struct Piece {
 // to the table's reach with the error reported.
 __device__ __forceinline__ int32_t load_len(const AttnArgs &a, int s, int32_t *raw_out)
 {
-    const int32_t raw = a.sync_table ? a.sync_words[s] : ld_prior(a.ctx_lens + s, a.chain == 2);
+    const int32_t raw = a.sync_table ? a.sync_words[s] : ld_prior(a.ctx_lens + s, a.chain >= 2);
     const int32_t cap = a.max_blocks * a.bs;
     *raw_out = raw;
     if (raw < 0 || raw > cap) {
@@ -586,7 +594,7 @@ __device__ __forceinline__ int32_t table_entry(const AttnArgs &a, int64_t idx)
         for (int j = 0; j < a.sync_npatch; ++j)
             if (pw[2 * j] == idx) return pw[2 * j + 1];
     }
-    return ld_prior(a.table + idx, a.chain == 2);
+    return ld_prior(a.table + idx, a.chain >= 2);
 }
 
 // Pool row of unit u's K tile (TMA y coordinate; V is Hkv*bs rows further),
@@ -681,12 +689,22 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // parameters (fused table sync) and no shared prefix, the first prologue
     // below reads nothing that another grid writes and writes only shared
     // memory, so a grid alone runs it before its wait, beside the grid
-    // before it (`early`).
-    const bool early = a.sync_table != nullptr && a.skip == nullptr && a.chain == 0;
+    // before it (`early`).  After a combine (chain 3) nothing before that
+    // combine is still running: the kernel reads and writes the table, the
+    // lengths and the pool at once, and each thread waits for the combine
+    // (`ready`) before it first writes the output or the workspace.
+    const bool early = a.sync_table != nullptr && a.skip == nullptr && (a.chain == 0 || a.chain == 3);
     if (a.chain != 1) grid_launch_dependents();
-    if (a.chain != 2 && !early) grid_dependency_wait();
+    if (a.chain <= 1 && !early) grid_dependency_wait();
     if (a.chain == 1) grid_launch_dependents();
-    const bool chained = a.chain == 2;
+    const bool chained = a.chain >= 2;
+    bool ready = a.chain != 3;  // the output and the workspace may be written
+    auto make_ready = [&]() {
+        if (!ready) {
+            grid_dependency_wait();
+            ready = true;
+        }
+    };
     auto write_sync = [&]() {
         // fused table sync: the grids before have completed (the wait
         // before this), and no CTA of this grid reads what is written here
@@ -732,12 +750,13 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
             T[S] = tot;
         }
         if (early) {
-            grid_dependency_wait();
+            if (a.chain == 0) grid_dependency_wait();
             write_sync();
         }
         for (int s = lo; s < hi; ++s) {  // sequences with no tile: writes after any wait
             const int32_t n = NL[s] & 0x7fffffff, ne = n - SK[s];
             if (ne != 0 || (s % a.P) != (int)blockIdx.x) continue;
+            make_ready();
             // the fused append needs the new token outside a shared prefix
             if (a.skip && a.k_new && n > 0) report(a.err, KV_ERR_DEVICE_BOUNDS);
             // an empty context has no softmax: its output is defined as
@@ -894,6 +913,7 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
         const bool split = p_first != p_last || pc.skip > 0;
         uint16_t *orow = a.out + ((int64_t)pc.s * Hq + (int64_t)pc.g * G) * D;
         float *slot = a.ws_part + ((int64_t)r + part) * MF;
+        make_ready();
         comp.store(orow, slot, split, lane);
         if (part == p_first && lane == 0)  // each run has one first part: it tells the combine
             a.ws_run[r] = make_int2(p_first, split ? p_last - p_first + 1 : 0);
@@ -981,10 +1001,12 @@ combine_kernel(const __grid_constant__ CombineArgs c)
     const int NG = (int)blockDim.x / NCT;  // groups of NCT threads
     extern __shared__ float4 s_dyn[];      // [CPT][blockDim] O, then M, then L (when NG > 1)
     const int r = blockIdx.x;
-    // the next grid in the stream may be scheduled now; it waits for this
-    // one to complete before touching anything this grid reads
-    grid_launch_dependents();
     grid_dependency_wait();  // the attention grid's partials and run table
+    // Release the next grid only now, when every grid before this one has
+    // completed: a decode grid that follows without a wait of its own (step
+    // overlap) relies on it, and until its own wait writes nothing that this
+    // grid reads or writes.
+    grid_launch_dependents();
     const int2 info = c.ws_run[r];
     const int s = r / c.Hkv, g = r % c.Hkv;
     const int npre = (c.skip != nullptr && c.skip[s] > 0) ? c.KS : 0;

@@ -7,6 +7,7 @@
 #include <atomic>
 
 #include "cascade_impl.cuh"
+#include "stream_order.h"
 
 namespace kvp {
 
@@ -84,7 +85,10 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (what != kLaunchCombine && cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
+    if (what != kLaunchCombine) {
+        if (cudaLaunchKernelEx(&cfg, fn, *tmap, a) != cudaSuccess) return KV_ERR_CUDA;
+        kvp_note_stream(st, false);
+    }
     if (what == kLaunchAttention) return KV_OK;
     CombineArgs c{a.out, a.ws_run, a.ws_part, a.S, a.Hkv, a.skip, a.ws_pre, a.KS};
     cudaLaunchConfig_t ccfg = cfg;
@@ -98,13 +102,17 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
         if (groups == 1) {
             ccfg.blockDim = dim3((unsigned)CombineShape<D, G, 2>::NCT);
             ccfg.dynamicSmemBytes = 0;
-            return cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 2>, c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+            if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 2>, c) != cudaSuccess) return KV_ERR_CUDA;
+            kvp_note_stream(st, true);
+            return KV_OK;
         }
     }
     const int threads = groups * (G * D / 4);
     ccfg.blockDim = dim3((unsigned)threads);
     ccfg.dynamicSmemBytes = combine_smem_bytes<D, G, 1>(threads);
-    return cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 1>, c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 1>, c) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(st, true);
+    return KV_OK;
 }
 
 // Shared-prefix kernel: with launch = false only reports the CTAs that fit
@@ -138,7 +146,9 @@ int cascade_run(const CUtensorMap *tmap, const CascadeArgs *c, int grid, int sm_
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, fn, *tmap, *c) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    if (cudaLaunchKernelEx(&cfg, fn, *tmap, *c) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(st, false);
+    return KV_OK;
 }
 
 }  // namespace kvp

@@ -17,6 +17,44 @@
 #include "pool_internal.h"
 #include "seqtab_internal.h"
 
+// ---- stream_order.h: the library's latest launch per stream.  A small table
+// (streams in use at once are few); a stream that fell out of it reads as
+// "not after a combine", the safe answer.
+namespace {
+constexpr int kStreamSlots = 64;
+struct StreamNote {
+    void *stream;
+    bool combine;
+    uint64_t stamp;
+};
+std::mutex g_stream_mu;
+StreamNote g_streams[kStreamSlots];
+uint64_t g_stream_clock = 0;
+}  // namespace
+
+void kvp_note_stream(void *stream, bool combine)
+{
+    std::lock_guard<std::mutex> lk(g_stream_mu);
+    int slot = -1, oldest = 0;
+    for (int i = 0; i < kStreamSlots; ++i) {
+        if (g_streams[i].stamp && g_streams[i].stream == stream) {
+            slot = i;
+            break;
+        }
+        if (g_streams[i].stamp < g_streams[oldest].stamp) oldest = i;
+    }
+    if (slot < 0) slot = oldest;
+    g_streams[slot] = StreamNote{stream, combine, ++g_stream_clock};
+}
+
+bool kvp_stream_after_combine(void *stream)
+{
+    std::lock_guard<std::mutex> lk(g_stream_mu);
+    for (int i = 0; i < kStreamSlots; ++i)
+        if (g_streams[i].stamp && g_streams[i].stream == stream) return g_streams[i].combine;
+    return false;
+}
+
 namespace {
 
 // Append: the decode step writes the new token's K and V before attending
@@ -224,7 +262,9 @@ int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_pl
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, cascade_plan_kernel<W>, *p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    if (cudaLaunchKernelEx(&cfg, cascade_plan_kernel<W>, *p) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(st, false);
+    return KV_OK;
 }
 
 // words the plan kernel carries: the plan's, plus the sync's lengths and
@@ -296,6 +336,7 @@ int kv_append(kv_pool *p, int layout, const uint16_t *k_new, const uint16_t *v_n
         (uint8_t *)p->desc.device_base, reinterpret_cast<const uint4 *>(k_new), reinterpret_cast<const uint4 *>(v_new),
         dev_table, dev_ctx_lens, p->desc.device_error, S, L.num_kv_heads, L.head_dim, p->desc.block_size, max_blocks,
         (int64_t)p->page_bytes, p->n_pages, p->pages_per_block[layout]);
+    kvp_note_stream(stream, false);
     return cudaGetLastError() == cudaSuccess ? KV_OK : KV_ERR_CUDA;
 }
 
@@ -404,6 +445,10 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
                 a.sync_words[nl + 2 * j + 1] = t->table[(size_t)idx];
             }
         }
+        // right after one of this library's combines on the stream, and with
+        // the pool's step overlap on, the decode grid starts while that
+        // combine finishes (chain 3)
+        if (p->step_overlap && kvp_stream_after_combine(stream)) a.chain = 3;
         rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                       kvp::kLaunchBoth, &P);
         if (rc || !sync) return rc;

@@ -14,6 +14,7 @@
 #include <cuda_runtime.h>
 
 #include "pool_internal.h"
+#include "stream_order.h"
 
 namespace {
 
@@ -308,6 +309,13 @@ int kv_set_attn_variant(kv_pool *p, int variant)
     return KV_OK;
 }
 
+int kv_set_attn_step_overlap(kv_pool *p, int on)
+{
+    if (!p || on < 0 || on > 1) return KV_ERR_INVALID_ARG;
+    p->step_overlap = on != 0;
+    return KV_OK;
+}
+
 int kv_block_table_upload(kv_pool *p, int layout, const int32_t *host_table, int S, int max_blocks,
                           const int32_t *host_ctx_lens, int32_t *dev_table, int32_t *dev_ctx_lens,
                           void *stream)
@@ -331,6 +339,7 @@ int kv_block_table_upload(kv_pool *p, int layout, const int32_t *host_table, int
     if (cudaMemcpyAsync(dev_ctx_lens, host_ctx_lens, sizeof(int32_t) * (size_t)S,
                         cudaMemcpyHostToDevice, st) != cudaSuccess)
         return KV_ERR_CUDA;
+    kvp_note_stream(stream, false);
     return KV_OK;
 }
 
@@ -342,6 +351,7 @@ int kv_pool_get_error(kv_pool *p, void *stream, int32_t *host_code)
         cudaSuccess)
         return KV_ERR_CUDA;
     if (cudaMemsetAsync(p->desc.device_error, 0, sizeof(int32_t), st) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(stream, false);
     return KV_OK;
 }
 
@@ -350,6 +360,7 @@ int kv_workspace_clear(void *workspace, size_t ws_bytes, void *stream)
     if (!workspace && ws_bytes) return KV_ERR_INVALID_ARG;
     if (!ws_bytes) return KV_OK;
     if (cudaMemsetAsync(workspace, 0, ws_bytes, (cudaStream_t)stream) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(stream, false);
     return KV_OK;
 }
 

@@ -49,6 +49,7 @@ struct kv_pool {
     int device = 0;
     int sm_count = 0;
     int attn_variant = 0;
+    bool step_overlap = false;                // kv_set_attn_step_overlap
     CUtensorMap tmap[KV_MAX_LAYOUTS];        // pool viewed as rows of d bf16, per layout
     bool tmap_ok[KV_MAX_LAYOUTS] = {false, false, false, false};
     kv_vmm_state vmm;

@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 
 #include "seqtab_internal.h"
+#include "stream_order.h"
 
 namespace {
 
@@ -63,7 +64,9 @@ int launch_chunk(kv_seqtab *t, int32_t *dev_table, int32_t *dev_lens, size_t li,
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, seqtab_sync_kernel<WORDS>, p) == cudaSuccess ? KV_OK : KV_ERR_CUDA;
+    if (cudaLaunchKernelEx(&cfg, seqtab_sync_kernel<WORDS>, p) != cudaSuccess) return KV_ERR_CUDA;
+    kvp_note_stream(st, false);
+    return KV_OK;
 }
 
 // parameter blocks of three sizes: a launch's cost grows with its parameter
@@ -86,6 +89,7 @@ extern "C" int kv_seqtab_sync(kv_seqtab *t, int32_t *dev_table, int32_t *dev_ctx
         if (cudaMemcpyAsync(dev_table, t->table.data(), total * sizeof(int32_t), cudaMemcpyHostToDevice, st) !=
             cudaSuccess)
             return KV_ERR_CUDA;
+        kvp_note_stream(st, false);
         t->counters.entries_uploaded += (int64_t)total;
         for (int32_t idx : t->changed) t->pending[(size_t)idx] = 0;
         t->changed.clear();

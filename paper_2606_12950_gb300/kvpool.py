@@ -180,6 +180,7 @@ def lib() -> ctypes.CDLL:
             "paged_decode_attn_seqtab": [P, P, P, P, P, P, P, P, I, I, F, I, P, SZ, P],
             "paged_decode_attn_multi": [P, I, P, P],
             "kv_set_attn_variant": [P, I],
+            "kv_set_attn_step_overlap": [P, I],
             "kv_cascade_workspace_bytes": [P, I, I, I, I, ctypes.POINTER(SZ)],
             "kv_pool_create_vmm": [ctypes.POINTER(kv_pool_desc), ctypes.POINTER(kv_vmm_desc), ctypes.POINTER(P)],
             "kv_pool_get_base": [P, ctypes.POINTER(P)],
@@ -522,6 +523,12 @@ def paged_decode_attn_cascade_seqtab(pool, seqtab, q, k_new, v_new, out, dev_tab
 
 def kv_set_attn_variant(pool, variant: int) -> None:
     _check("kv_set_attn_variant", lib().kv_set_attn_variant(pool, int(variant)))
+
+
+def kv_set_attn_step_overlap(pool, on: bool) -> None:
+    """Let a decode kernel start while the previous attention call's combine
+    on the same stream finishes (see kvpool.h)."""
+    _check("kv_set_attn_step_overlap", lib().kv_set_attn_step_overlap(pool, int(bool(on))))
 
 
 # ------------------------------------------------------------ sequence tables

@@ -51,6 +51,9 @@ class DevicePool:
     def set_variant(self, v: int) -> None:
         K.kv_set_attn_variant(self.handle, v)
 
+    def set_step_overlap(self, on: bool) -> None:
+        K.kv_set_attn_step_overlap(self.handle, on)
+
     def close(self) -> None:
         if self.handle:
             K.kv_pool_destroy(self.handle)
@@ -121,6 +124,9 @@ class VmmPool:
 
     def set_variant(self, v: int) -> None:
         K.kv_set_attn_variant(self.handle, v)
+
+    def set_step_overlap(self, on: bool) -> None:
+        K.kv_set_attn_step_overlap(self.handle, on)
 
     def close(self) -> None:
         if self.handle:
