@@ -718,8 +718,9 @@ def main():
     iso_gbs = float(np.mean(iso_bytes)) / (iso_ms * 1e-3) / 1e9
     peak, peak_kind = load_peaks()
     if cascade is not None:
-        step_kernels = ("seqtab_sync_kernel, cascade_plan_kernel, paged_attn_kernel (suffixes, fused append) "
-                        "beside cascade_prefix_kernel, combine_kernel")
+        step_kernels = (("cascade_plan_kernel (with the table sync)" if runner.cascade_sync else
+                         "seqtab_sync_kernel, cascade_plan_kernel")
+                        + ", paged_attn_kernel (suffixes, fused append) beside cascade_prefix_kernel, combine_kernel")
     elif args.separate_append:
         step_kernels = "seqtab_sync_kernel, append_kernel, paged_attn_kernel, combine_kernel"
     elif multi:
