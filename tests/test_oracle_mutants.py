@@ -37,6 +37,10 @@ MUTANTS = {
     "layout head/offset transposed": ("return block * page_elems + (((int64_t)which * Hkv + g) * bs + off) * d + c;",
                                       "return block * page_elems + (((int64_t)which * bs + off) * Hkv + g) * d + c;"),
     "combine weight sign": ("double w = exp(m[i] - M);", "double w = exp(M - m[i]);"),
+    "split combine drops the last split": ("for (int i = 0; i < ns; ++i) {\n                double w",
+                                           "for (int i = 0; i + 1 < ns; ++i) {\n                double w"),
+    "splits overlap by one key": ("int end = start + split_len < n ? start + split_len : n;",
+                                  "int end = start + split_len + 1 < n ? start + split_len + 1 : n;"),
     "combine denominator without l": ("denom += w * l[i];", "denom += w;"),
 }
 
@@ -48,15 +52,15 @@ def _pin_calls():
             continue
         marks = getattr(fn, "pytestmark", [])
         params = [m for m in marks if m.name == "parametrize"]
-        sig = inspect.signature(fn).parameters
-        if params:
-            argnames, values = params[0].args
+        # every combination of every parametrize mark, as pytest runs them
+        combos = [{}]
+        for m in params:
+            argnames, values = m.args
             argnames = [a.strip() for a in argnames.split(",")]
-            for v in values:
-                v = v if isinstance(v, tuple) else (v,)
-                calls.append((name, fn, dict(zip(argnames, v))))
-        else:
-            calls.append((name, fn, {}))
+            combos = [dict(c, **dict(zip(argnames, v if isinstance(v, tuple) else (v,))))
+                      for c in combos for v in values]
+        for kw in combos:
+            calls.append((name, fn, kw))
     out = []
     for name, fn, kw in calls:
         if "oracle_mod" in sig_of(fn):

@@ -204,6 +204,58 @@ def test_split_combine_equals_unsplit(oracle_mod, split_len):
     np.testing.assert_allclose(split, full, rtol=0, atol=1e-13)
 
 
+@pytest.mark.parametrize("seed,lens,Hq,Hkv,d,bs", CASES)
+@pytest.mark.parametrize("split_len", [1, 2, 5, 16])
+def test_split_attention_equals_dense_brute_force(oracle_mod, seed, lens, Hq, Hkv, d, bs, split_len):
+    """The split-K form (per-split partials, then the combine step) pinned
+    directly to the numpy gather and softmax, not only to the unsplit
+    oracle: a wrong rescale between splits, a dropped split or a merge in
+    the wrong order fails here."""
+    b = tiny_random(seed, lens, Hq, Hkv, d, bs)
+    got = oracle_mod.split_attention(b.pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q,
+                                     b.table, b.ctx_lens, b.scale, split_len)
+    for s, (K, V) in enumerate(gather_dense(b, b.pool)):
+        q = W.bf16_bits_to_f64(b.q[s])
+        np.testing.assert_allclose(got[s], numpy_attention(q, K, V, b.scale), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("split_len", [1, 3, 4])
+def test_split_attention_with_identical_keys_gives_mean_of_v(oracle_mod, split_len):
+    """Closed form through the split path: equal keys make every score equal,
+    so each split's partial and their merge must give the plain mean of V."""
+    b = tiny_random(25, [9, 13], Hq=4, Hkv=2, d=8, bs=4)
+    pool = b.pool.copy()
+    rng = np.random.default_rng(6)
+    for s in range(b.S):
+        n = int(b.ctx_lens[s])
+        for g in range(b.Hkv):
+            _set_rows(b, pool, s, g, 0, [W.bf16_normal(rng, (b.d,))] * n)
+    got = oracle_mod.split_attention(pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q, b.table,
+                                     b.ctx_lens, b.scale, split_len)
+    for s, (K, V) in enumerate(gather_dense(b, pool)):
+        for h in range(b.Hq):
+            np.testing.assert_allclose(got[s, h], V[h // b.G].mean(axis=0), rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("seed,lens,Hq,Hkv,d,bs", CASES)
+def test_sequence_subset_equals_dense_brute_force(oracle_mod, seed, lens, Hq, Hkv, d, bs):
+    """The seq_ids subset path pinned directly: the requested sequences'
+    rows equal the numpy gather and softmax, every other row stays NaN, and
+    the order of the ids does not matter."""
+    b = tiny_random(seed, lens, Hq, Hkv, d, bs)
+    ids = np.array([s for s in range(b.S) if s % 2 == 1][::-1] + [0], dtype=np.int32)
+    got = oracle_mod.paged_attention(b.pool, b.n_pages, b.page_elems, b.bs, b.Hkv, b.d, b.q, b.table,
+                                     b.ctx_lens, b.scale, seq_ids=ids)
+    dense = gather_dense(b, b.pool)
+    for s in range(b.S):
+        if s in set(ids.tolist()):
+            K, V = dense[s]
+            q = W.bf16_bits_to_f64(b.q[s])
+            np.testing.assert_allclose(got[s], numpy_attention(q, K, V, b.scale), rtol=0, atol=1e-12)
+        else:
+            assert np.isnan(got[s]).all()
+
+
 def test_append_writes_exactly_the_new_slot(oracle_mod):
     b = W.make_batch(31, [17, 64, 100, 255, 0], Hq=4, Hkv=2, d=64, bs=16, n_pages=128,
                      pool_fill="sentinel")
