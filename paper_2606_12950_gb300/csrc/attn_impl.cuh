@@ -947,18 +947,20 @@ constexpr int kCombineBatch = 8;  // records each thread loads per round trip
 
 // Thread groups per combine CTA (a run's records are spread over the
 // groups, kCombineBatch loads in flight per thread): enough groups for
-// about 8 records per thread, up to 1024 threads, and at least 256 threads,
-// so that the longest runs of a heavy-tailed batch (tens of records) take
-// few round trips; at 64 registers four 256-thread CTAs fit on an SM, one
-// wave covering 600 runs.  In shared-prefix mode every member run carries
-// the KS prefix records and the parts of a short suffix, so the counts are
-// uniform and small: there the minimum is 128 threads, one group when a
-// run's output has 128 float4 columns or more.
+// about 8 records per thread, up to 1024 threads, and at least 128 threads
+// (one group when a run's output has 128 float4 columns or more).  Small
+// CTAs leave room on the SMs for the next step's decode CTAs, which start
+// as the combine's CTAs finish: on the Llama-3-8B-shaped layer (64
+// sequences, 32 q / 8 KV heads) 128-thread CTAs took 54.5-54.9 µs per step
+// against 55.1-55.4 with 256 (six same-box pairs), at a cost of about 1 µs
+// in 296 for three co-located models, whose heavy-tailed runs take more
+// round trips with one group.
 template <int D, int G>
 inline int combine_groups(double records_per_run, bool shared_prefix)
 {
     constexpr int NC = G * D / 4;
-    const int floor_threads = shared_prefix ? 128 : 256;
+    (void)shared_prefix;
+    const int floor_threads = 128;
     const int base = NC >= floor_threads ? 1 : floor_threads / NC;
     const int most = kCombineMaxThreads / NC;
     int want = (int)(records_per_run / 8.0 + 0.999);

@@ -98,8 +98,9 @@ int attn_run(const CUtensorMap *tmap, AttnArgs a, int P_req, int sm_count, cudaS
     const int groups = combine_groups<D, G>(per_run, a.skip != nullptr);
     ccfg.gridDim = dim3((unsigned)(a.S * a.Hkv));
     if constexpr (G * D / 4 >= 128) {
-        // one group: two columns a thread, so that every run fits in one wave
-        if (groups == 1) {
+        // one group in shared-prefix mode: two columns a thread, so that
+        // every member run fits in one wave
+        if (groups == 1 && a.skip != nullptr) {
             ccfg.blockDim = dim3((unsigned)CombineShape<D, G, 2>::NCT);
             ccfg.dynamicSmemBytes = 0;
             if (cudaLaunchKernelEx(&ccfg, combine_kernel<D, G, 2>, c) != cudaSuccess) return KV_ERR_CUDA;
