@@ -205,3 +205,37 @@ def test_seqtab_attention_argument_checks_precede_any_launch():
                                        args["dev_table"], args["dev_lens"], args["S"], 32, 0.1, 0, fake, 1 << 20)
         assert e.value.code == code, over
     t.close()
+
+
+def test_cascade_seqtab_argument_checks_precede_any_launch():
+    h, _ = make_pool(n_pages=16)
+    h2, _ = make_pool(n_pages=16)
+    t = K.SeqTab(h, 0, 4, 8)
+    fake = 1 << 41  # never dereferenced: every call below fails its host checks
+    plan = K.PrefixPlan([([0, 1], 64)])
+    cases = [
+        (h2, t, dict(S=4), K.KV_ERR_INVALID_ARG),                  # table over another pool
+        (h, t, dict(S=5), K.KV_ERR_INVALID_ARG),                   # more rows than the table has
+        (h, t, dict(S=4, dev_table=None), K.KV_ERR_INVALID_ARG),   # no device table
+        (h, t, dict(S=4, v_new=None), K.KV_ERR_INVALID_ARG),       # k_new without v_new
+    ]
+    for pool, tab, over, code in cases:
+        args = dict(q=fake, k_new=fake, v_new=fake, out=fake, dev_table=fake, dev_lens=fake, S=4)
+        args.update(over)
+        with pytest.raises(K.KVError) as e:
+            K.paged_decode_attn_cascade_seqtab(pool, tab, args["q"], args["k_new"], args["v_new"], args["out"],
+                                               args["dev_table"], args["dev_lens"], args["S"], 32, 0.1, plan,
+                                               fake, 1 << 20)
+        assert e.value.code == code, over
+    rc = K.lib().paged_decode_attn_cascade_seqtab(h, t.handle, fake, fake, fake, fake, fake, fake, 4, 32,
+                                                  0.1, None, -1, None, fake, 1 << 20, None)
+    assert rc == K.KV_ERR_INVALID_ARG  # a negative group count
+    t.close()
+
+
+def test_step_overlap_switch_checks_its_arguments():
+    h, _ = make_pool(n_pages=16)
+    K.kv_set_attn_step_overlap(h, True)
+    K.kv_set_attn_step_overlap(h, False)
+    assert K.lib().kv_set_attn_step_overlap(h, 2) == K.KV_ERR_INVALID_ARG
+    assert K.lib().kv_set_attn_step_overlap(None, 1) == K.KV_ERR_INVALID_ARG
