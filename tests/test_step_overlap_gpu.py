@@ -101,3 +101,52 @@ def test_step_overlap_gives_the_bits_of_waiting_steps(between, num_splits):
     for pool, t, _ in (on, off):
         t.close()
         pool.close()
+
+
+def test_step_overlap_with_host_buffers():
+    """The end-to-end form the benchmark times: q, k_new, v_new and out in
+    pinned host memory that the kernels read and write directly, steps back
+    to back with the overlap on; the same bits as device buffers with the
+    overlap off."""
+    steps = 6
+    b = W.config2_llama8b(steps=steps + 8)
+    on = _side(b, True, steps, 0)
+    off = _side(b, False, steps, 0)
+    pool_on, _, buf_on = on
+    hin = torch.empty(buf_on.inputs.shape, dtype=torch.bfloat16).pin_memory()
+    hin.copy_(buf_on.inputs.view(torch.bfloat16).cpu())
+    hout = torch.full(buf_on.out.shape, float("nan"), dtype=torch.bfloat16).pin_memory()
+    buf_on.io(hin, hout)
+    _run(on, steps, None)
+    _run(off, steps, None)
+    assert torch.equal(hout.view(torch.int16), off[2].out.cpu().view(torch.int16))
+    assert np.array_equal(pool_on.download(), off[0].download())
+    assert pool_on.error() == 0 and off[0].error() == 0
+    for pool, t, _ in (on, off):
+        t.close()
+        pool.close()
+
+
+def test_step_overlap_on_two_streams():
+    """Two batches on two streams, their steps interleaved on the host with
+    the overlap on: each stream's record of the library's last launch is its
+    own, so each batch gives the bits it gives alone with the overlap off."""
+    steps = 6
+    b = W.config2_llama8b(steps=steps + 8)
+    sides = [_side(b, True, steps, 0), _side(b, True, steps, 0)]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    torch.cuda.synchronize()
+    for i in range(steps):
+        for (pool, t, buf), st in zip(sides, streams):
+            t.advance()
+            buf.sync_append_attend(t, st)
+    torch.cuda.synchronize()
+    ref = _side(b, False, steps, 0)
+    _run(ref, steps, None)
+    for pool, t, buf in sides:
+        assert torch.equal(buf.out.view(torch.int16), ref[2].out.view(torch.int16))
+        assert np.array_equal(pool.download(), ref[0].download())
+        assert pool.error() == 0
+    for pool, t, _ in sides + [ref]:
+        t.close()
+        pool.close()
