@@ -9,8 +9,10 @@ overlap on and one with it off: steps back to back on one stream (only the
 final output and the pool are compared, since any copy between the steps
 would separate them), steps with an output copy between them, steps with
 the pool's error read between them (a library copy, which turns the
-overlap off for the next call), and automatic and forced split counts.
-The final output is checked against the fp64 oracle, every sequence.
+overlap off for the next call), and automatic and forced split counts;
+also pinned host buffers (the benchmark's end-to-end form) and two batches
+on two streams with their steps interleaved.  The final output is checked
+against the fp64 oracle, every sequence.
 """
 import numpy as np
 import pytest
