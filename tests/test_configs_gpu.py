@@ -50,7 +50,7 @@ def _check_all(got, host_pool, n_pages, page_elems, bs, Hkv, d, q, table, lens, 
 
 
 def _run_chains(n_chains, steps, median, max_out, seed=1003, check_every=1, cascade=False,
-                until_stage_end=False, sync_in_call=False, bits=None):
+                until_stage_end=False, sync_in_call=False, bits=None, pages_per_chain=150):
     """Agent chains driven as the benchmark drives them: the sequence table's
     sync, then the cascade call with the fused append (shared-prefix mode;
     with sync_in_call one paged_decode_attn_cascade_seqtab call, the sync
@@ -64,7 +64,7 @@ def _run_chains(n_chains, steps, median, max_out, seed=1003, check_every=1, casc
 
     d, Hq, Hkv, bs = 128, 32, 8, 16
     max_blocks = (W.PREFIX_TOKENS + 4 * max_out * 2) // bs + 8
-    n_pages = 128 + n_chains * 150 + 64  # about twice the expected need
+    n_pages = 128 + n_chains * pages_per_chain + 64  # about twice the expected need
     page_elems = 2 * Hkv * bs * d
     host_pool = np.empty(n_pages * page_elems, np.uint16)
     W.bf16_normal_fill(host_pool, seed + 7919)
@@ -155,6 +155,23 @@ def test_table_sync_carried_by_the_plan_kernel_gives_the_separate_sync_bits():
             assert np.array_equal(a, b), i
     assert fused[0][3] >= 1 and fused[-1][3] == fused[0][3]  # no sync kernel after the first step
     assert separate[-1][3] >= separate[0][3] + 39
+
+
+def test_table_sync_too_large_for_the_plan_kernel_runs_first():
+    """1500 chains: the plan (about 3000 words) and the table's 1501 lengths
+    exceed the plan kernel's 4080-word block, so paged_decode_attn_cascade_seqtab
+    runs the sync kernel first on every step; the bits still equal the
+    separate sync followed by the cascade call, and the run matches the
+    oracle on the first and last of six steps."""
+    fused, separate = [], []
+    _run_chains(1500, steps=6, median=5.0, max_out=40, check_every=5, cascade=True, sync_in_call=True,
+                bits=fused, pages_per_chain=16)
+    _run_chains(1500, steps=6, median=5.0, max_out=40, check_every=5, cascade=True, bits=separate,
+                pages_per_chain=16)
+    for i, (f, r) in enumerate(zip(fused, separate)):
+        for a, b in zip(f[:3], r[:3]):
+            assert np.array_equal(a, b), i
+    assert fused[-1][3] >= fused[0][3] + 5  # a sync kernel on every step
 
 
 def test_agent_chains_stage_turnover_cascade():
