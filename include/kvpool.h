@@ -103,6 +103,8 @@ typedef struct kv_stats {
     uint64_t bytes_used;                     /* sum of used blocks' bytes */
     uint64_t bytes_total;                    /* pages_total * page_bytes */
     uint64_t bytes_mapped;                   /* physically backed bytes (VMM pool); bytes_total otherwise */
+    int64_t attn_calls_overlapped;           /* attention calls that started while the previous
+                                                call's combine finished (kv_set_attn_step_overlap) */
 } kv_stats;
 
 /* ---------------------------------------------------------------- pool --- */
@@ -605,7 +607,8 @@ int paged_decode_attn_multi(kv_pool *pool, int n, const kv_attn_batch *batches, 
  * the workspace:
  *     3 * n_groups + 2 + (members) + S <= 4080 words.
  * Workspace: kv_cascade_workspace_bytes() (256-byte aligned); nothing in it
- * needs initialising.
+ * needs initialising.  Consecutive calls on one workspace alternate between
+ * its two skip arrays (step overlap, kv_set_attn_step_overlap).
  * Errors: KV_ERR_INVALID_ARG (bad plan, duplicate member, words over the
  * limit), KV_ERR_WORKSPACE, KV_ERR_UNSUPPORTED, KV_ERR_CUDA; on the device a
  * member shorter than its prefix sets KV_ERR_DEVICE_BOUNDS in the error word.
@@ -693,14 +696,26 @@ int kv_set_attn_variant(kv_pool *pool, int variant);
  * and starts streaming at once, and waits for the combine before it writes
  * the output or the workspace.  That is safe because the combine releases
  * the next kernel only after everything before it in the stream has
- * completed.  Any other launch or copy of this library on the stream in
- * between (a table sync, an append, an upload) turns it off for the next
- * call, and so does a stream the library has not seen.  Results are the
- * same bits either way.  The caller's side of the contract: work of
+ * completed.  A shared-prefix call (paged_decode_attn_cascade,
+ * paged_decode_attn_cascade_seqtab) overlaps the combine of the previous
+ * shared-prefix call when that call used the same workspace with the same
+ * layout: its plan kernel writes the plan, the skips (into the workspace's
+ * other skip array) and the table sync at once and raises a flag in the
+ * workspace; the decode kernel over the suffixes, released by the prefix
+ * kernel before that kernel's own wait, reads after that flag and writes
+ * its output and partials after a second flag, which the plan kernel
+ * raises once the combine has completed.  Any other launch or copy of this
+ * library on the stream in between (a table sync, an append, an upload)
+ * turns it off for the next call, and so does a stream the library has not
+ * seen.  Results are the same bits either way; kv_pool_stats counts the
+ * calls that overlapped.  The caller's side of the contract: work of
  * others between two attention calls on one stream must not be launched as
  * a programmatic dependent that releases its own dependents before it has
- * finished writing (ordinary kernels and copies are fine), and one host
- * thread submits to the stream at a time.
+ * finished writing (ordinary kernels and copies are fine); one host thread
+ * submits to the stream at a time; and the earlier call's workspace and
+ * output are not handed to the later call as its table, lengths or inputs
+ * (a stream-ordered allocator that reuses freed memory on the same stream
+ * at once can do that when they are freed between the calls).
  */
 int kv_set_attn_step_overlap(kv_pool *pool, int on);
 

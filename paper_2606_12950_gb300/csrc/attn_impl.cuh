@@ -127,8 +127,18 @@ struct AttnArgs {
     // of this library, which released this grid only after its own wait, so
     // every grid before that combine has completed (release, no wait at the
     // start, a wait before the first write of the output or the workspace,
-    // which the combine still uses, and at every exit)
+    // which the combine still uses, and at every exit); 4 beside the
+    // shared-prefix kernel while the previous step's shared-prefix combine
+    // finishes (release, no wait at the start; the plan kernel's two flags,
+    // below, stand in for the waits: the first before anything the plan
+    // kernel writes is read, the second before the first write of the output
+    // or the workspace; a wait for the prefix grid at every exit)
     int32_t chain;
+    // chain 4: the plan kernel sets flags[0] = epoch once the plan, the
+    // skips and the table sync are written, and flags[1] = epoch once every
+    // grid before it has completed
+    const uint64_t *flags;
+    uint64_t epoch;
     // fused table sync (paged_decode_attn_seqtab): this step's lengths of
     // rows [0, sync_nlens) and its changed table entries travel here.  The
     // kernel takes the lengths and those entries from here, and the CTAs
@@ -154,6 +164,23 @@ __device__ __forceinline__ void wait_phase(uint32_t bar, uint32_t parity, int32_
         if ((it & 1023u) == 0 && global_timer_ns() - t0 > kWaitLimitNs) {
             report(err, KV_ERR_DEVICE_TIMEOUT);
             dead = true;
+            return;
+        }
+    }
+}
+
+// bounded wait until another grid has stored `epoch` in *flag (release
+// store; this load acquires); a wait past the limit records
+// KV_ERR_DEVICE_TIMEOUT and returns
+__device__ __forceinline__ void wait_flag(const uint64_t *flag, uint64_t epoch, int32_t *err)
+{
+    if (ld_acquire_gpu(flag) == epoch) return;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 1;; ++it) {
+        __nanosleep(64);
+        if (ld_acquire_gpu(flag) == epoch) return;
+        if ((it & 255u) == 0 && global_timer_ns() - t0 > kWaitLimitNs) {
+            report(err, KV_ERR_DEVICE_TIMEOUT);
             return;
         }
     }
@@ -692,19 +719,30 @@ paged_attn_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constan
     // before it (`early`).  After a combine (chain 3) nothing before that
     // combine is still running: the kernel reads and writes the table, the
     // lengths and the pool at once, and each thread waits for the combine
-    // (`ready`) before it first writes the output or the workspace.
+    // (`ready`) before it first writes the output or the workspace.  Beside
+    // the prefix kernel of a step that overlaps the previous step's
+    // shared-prefix combine (chain 4), the plan kernel's flags take the place
+    // of those waits: the first before the lengths, skips and table are read,
+    // the second before the first write of the output or the workspace.
     const bool early = a.sync_table != nullptr && a.skip == nullptr && (a.chain == 0 || a.chain == 3);
     if (a.chain != 1) grid_launch_dependents();
     if (a.chain <= 1 && !early) grid_dependency_wait();
     if (a.chain == 1) grid_launch_dependents();
     const bool chained = a.chain >= 2;
-    bool ready = a.chain != 3;  // the output and the workspace may be written
+    bool ready = a.chain != 3 && a.chain != 4;  // the output and the workspace may be written
     auto make_ready = [&]() {
         if (!ready) {
-            grid_dependency_wait();
+            if (a.chain == 4)
+                wait_flag(a.flags + 1, a.epoch, a.err);
+            else
+                grid_dependency_wait();
             ready = true;
         }
     };
+    if (a.chain == 4) {
+        if (tid == 0) wait_flag(a.flags, a.epoch, a.err);
+        __syncthreads();
+    }
     auto write_sync = [&]() {
         // fused table sync: the grids before have completed (the wait
         // before this), and no CTA of this grid reads what is written here

@@ -58,7 +58,7 @@ struct CascadeArgs {
     int32_t n_groups;
     int32_t n_members;
     float qk_scale;       // scale * log2(e)
-    int32_t pad;
+    int32_t overlap;      // 1: release the decode grid before the wait (it waits on the plan kernel's flags)
     // the plan in the workspace, written by the plan kernel before this grid
     // reads it: [n_groups + 1] first row tile of each group | [n_groups + 1]
     // first member index | [n_groups] prefix tokens | [n_members] member
@@ -170,10 +170,14 @@ cascade_prefix_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_con
     // Wait for the grid before (the plan kernel; through it the table sync
     // and the previous step's combine), then release the decode kernel that
     // follows: it runs beside this grid on the SMs this grid leaves free and
-    // relies on this wait having completed in every CTA here.  The plan is
-    // read only after the wait: the plan kernel wrote it.
+    // relies on this wait having completed in every CTA here.  When the step
+    // overlaps the previous step's combine, the decode kernel waits on the
+    // plan kernel's flags instead and is released first.  The plan is read
+    // and the records written only after the wait: the plan kernel wrote the
+    // plan, and the previous combine read the records.
+    if (c.overlap) grid_launch_dependents();
     grid_dependency_wait();
-    grid_launch_dependents();
+    if (!c.overlap) grid_launch_dependents();
 
     const int32_t *tile_off = c.plan;
     const int32_t *mem_off = tile_off + c.n_groups + 1;

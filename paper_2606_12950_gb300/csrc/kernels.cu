@@ -5,6 +5,8 @@
 // batches as one chain (paged_decode_attn_multi) and shared-prefix
 // attention (paged_decode_attn_cascade).
 #include <algorithm>
+#include <atomic>
+#include <chrono>
 #include <cmath>
 #include <memory>
 #include <mutex>
@@ -26,6 +28,7 @@ struct StreamNote {
     void *stream;
     bool combine;
     uint64_t stamp;
+    KvpCascadeNote cascade;  // ws null: not a shared-prefix combine
 };
 std::mutex g_stream_mu;
 StreamNote g_streams[kStreamSlots];
@@ -44,7 +47,26 @@ void kvp_note_stream(void *stream, bool combine)
         if (g_streams[i].stamp < g_streams[oldest].stamp) oldest = i;
     }
     if (slot < 0) slot = oldest;
-    g_streams[slot] = StreamNote{stream, combine, ++g_stream_clock};
+    g_streams[slot] = StreamNote{stream, combine, ++g_stream_clock, KvpCascadeNote{}};
+}
+
+void kvp_note_cascade_combine(void *stream, const KvpCascadeNote &n)
+{
+    std::lock_guard<std::mutex> lk(g_stream_mu);
+    for (int i = 0; i < kStreamSlots; ++i)
+        if (g_streams[i].stamp && g_streams[i].stream == stream && g_streams[i].combine) g_streams[i].cascade = n;
+}
+
+bool kvp_stream_after_cascade(void *stream, KvpCascadeNote *n)
+{
+    std::lock_guard<std::mutex> lk(g_stream_mu);
+    for (int i = 0; i < kStreamSlots; ++i)
+        if (g_streams[i].stamp && g_streams[i].stream == stream) {
+            if (!g_streams[i].combine || !g_streams[i].cascade.ws) return false;
+            *n = g_streams[i].cascade;
+            return true;
+        }
+    return false;
 }
 
 bool kvp_stream_after_combine(void *stream)
@@ -193,6 +215,9 @@ struct PlanParams {
     int32_t *ws_skip;
     int32_t *sync_table;  // fused table sync: null for none
     int32_t *sync_lens;
+    uint64_t *flags;      // overlap: [0] set to epoch once everything is written, [1] once the grids before completed
+    uint64_t epoch;
+    int32_t overlap;
     int32_t n_words;      // plan words
     int32_t S;
     int32_t sync_nlens;
@@ -203,10 +228,17 @@ struct PlanParams {
 template <int W>
 __global__ void cascade_plan_kernel(const __grid_constant__ PlanParams<W> p)
 {
-    // the grids before (the previous step's kernels, which read the plan,
-    // the lengths and the table) have completed after this wait; the grid
-    // after waits for this one to complete before it reads any of them
-    kvp::grid_dependency_wait();
+    // Alone: the grids before (the previous step's kernels, which read the
+    // plan, the skips, the lengths and the table) have completed after this
+    // wait; the grid after waits for this one to complete before it reads
+    // any of them.  Overlapping the previous step's shared-prefix combine
+    // (overlap): that combine reads none of what is written here (its skips
+    // are the other of the workspace's two skip arrays), so everything is
+    // written at once and flags[0] tells the decode grid, which does not
+    // wait for this grid; flags[1] tells it when the combine has completed.
+    // The prefix grid still waits for this grid to complete, which is after
+    // the wait below.
+    if (!p.overlap) kvp::grid_dependency_wait();
     kvp::grid_launch_dependents();
     for (int i = threadIdx.x; i < p.n_words; i += blockDim.x) p.ws_plan[i] = p.words[i];
     const int32_t *skip = p.words + (p.n_words - p.S);
@@ -216,6 +248,38 @@ __global__ void cascade_plan_kernel(const __grid_constant__ PlanParams<W> p)
         for (int i = threadIdx.x; i < p.sync_nlens; i += blockDim.x) p.sync_lens[i] = lw[i];
         for (int j = threadIdx.x; j < p.sync_npatch; j += blockDim.x) p.sync_table[pw[2 * j]] = pw[2 * j + 1];
     }
+    if (!p.overlap) return;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        kvp::st_release_gpu(p.flags, p.epoch);
+        kvp::grid_dependency_wait();
+        kvp::st_release_gpu(p.flags + 1, p.epoch);
+    }
+}
+
+// a plan launch that overlaps the previous step's shared-prefix combine
+struct PlanOverlap {
+    bool on;
+    uint64_t *flags;
+    uint64_t epoch;
+};
+
+// A fresh 64-bit tag per overlapping call: the decode kernel takes a flag
+// as set only when it holds this call's tag, so a flag left by an earlier
+// call, or whatever the workspace held before, is never taken for it.
+// SplitMix64 (Steele, Lea and Flood, 2014) over a counter, salted per
+// process.
+uint64_t next_epoch()
+{
+    static std::atomic<uint64_t> ctr{0};
+    static const uint64_t salt =
+        (uint64_t)std::chrono::steady_clock::now().time_since_epoch().count() ^ (uint64_t)(uintptr_t)&ctr;
+    uint64_t z = salt + 0x9E3779B97F4A7C15ull * (ctr.fetch_add(1, std::memory_order_relaxed) + 1);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    z ^= z >> 31;
+    return z ? z : 1;
 }
 
 // parameter blocks of three sizes (a launch's host cost grows with its
@@ -225,12 +289,15 @@ constexpr int kPlanMidWords = 2040;
 
 template <int W>
 int cascade_plan_launch(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip,
-                        const FusedSync *sync, cudaStream_t st)
+                        const FusedSync *sync, const PlanOverlap &ov, cudaStream_t st)
 {
     static thread_local std::unique_ptr<PlanParams<W>> buf(new PlanParams<W>());
     PlanParams<W> *p = buf.get();
     p->ws_plan = ws_plan;
     p->ws_skip = ws_skip;
+    p->flags = ov.flags;
+    p->epoch = ov.epoch;
+    p->overlap = ov.on ? 1 : 0;
     p->n_words = n_words;
     p->S = S;
     std::copy(words, words + n_words, p->words);
@@ -275,15 +342,15 @@ inline size_t plan_sync_words(int n_words, const FusedSync *sync)
 }
 
 int cascade_plan_run(const int32_t *words, int n_words, int S, int32_t *ws_plan, int32_t *ws_skip,
-                     const FusedSync *sync, cudaStream_t st)
+                     const FusedSync *sync, const PlanOverlap &ov, cudaStream_t st)
 {
     const size_t n = plan_sync_words(n_words, sync);
     if (n <= (size_t)kPlanSmallWords)
-        return cascade_plan_launch<kPlanSmallWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
+        return cascade_plan_launch<kPlanSmallWords>(words, n_words, S, ws_plan, ws_skip, sync, ov, st);
     if (n <= (size_t)kPlanMidWords)
-        return cascade_plan_launch<kPlanMidWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
+        return cascade_plan_launch<kPlanMidWords>(words, n_words, S, ws_plan, ws_skip, sync, ov, st);
     if (n > (size_t)kvp::kCascadeWords) return KV_ERR_INVALID_ARG;  // the caller syncs separately first
-    return cascade_plan_launch<kvp::kCascadeWords>(words, n_words, S, ws_plan, ws_skip, sync, st);
+    return cascade_plan_launch<kvp::kCascadeWords>(words, n_words, S, ws_plan, ws_skip, sync, ov, st);
 }
 
 // workspace: per-run (first part, parts) as int2 (padded to 256 bytes),
@@ -295,15 +362,20 @@ size_t ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off)
     return hdr + kvp::attn_partial_slots(S, Hkv, P) * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
 
-// cascade workspace: the above, then the per-sequence skip (padded to 256
-// bytes), the plan words (kCascadeWords, padded), then kMaxKeySplits prefix
-// records per (sequence, KV head)
+// cascade workspace: the above, then two arrays of per-sequence skips (each
+// padded to 256 bytes; consecutive calls use different ones, so that a plan
+// kernel can write its skips while the previous step's combine still reads
+// the other), the plan kernel's two flags (256 bytes), the plan words
+// (kCascadeWords, padded), then kMaxKeySplits prefix records per (sequence,
+// KV head)
 size_t cascade_ws_layout(int S, int Hkv, int G, int D, int P, size_t *part_off, size_t *skip_off, size_t *pre_off,
-                         size_t *plan_off)
+                         size_t *plan_off, size_t *flags_off = nullptr)
 {
     const size_t base = (ws_layout(S, Hkv, G, D, P, part_off) + 255) / 256 * 256;
+    const size_t skip_bytes = ((size_t)S * 4 + 255) / 256 * 256;
     *skip_off = base;
-    *plan_off = base + ((size_t)S * 4 + 255) / 256 * 256;
+    if (flags_off) *flags_off = base + 2 * skip_bytes;
+    *plan_off = base + 2 * skip_bytes + 256;
     *pre_off = *plan_off + ((size_t)kvp::kCascadeWords * 4 + 255) / 256 * 256;
     return *pre_off + (size_t)kvp::kMaxKeySplits * S * Hkv * (size_t)((G * D + 2 * G + 3) / 4 * 4) * 4;
 }
@@ -448,7 +520,10 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         // right after one of this library's combines on the stream, and with
         // the pool's step overlap on, the decode grid starts while that
         // combine finishes (chain 3)
-        if (p->step_overlap && kvp_stream_after_combine(stream)) a.chain = 3;
+        if (p->step_overlap && kvp_stream_after_combine(stream)) {
+            a.chain = 3;
+            p->overlapped.fetch_add(1, std::memory_order_relaxed);
+        }
         rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                       kvp::kLaunchBoth, &P);
         if (rc || !sync) return rc;
@@ -506,8 +581,9 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         }
     }
     const int tiles = tile_off[ng];
-    size_t skip_off, pre_off, plan_off;
-    const size_t need = cascade_ws_layout(S, Hkv, G, L.head_dim, P, &part_off, &skip_off, &pre_off, &plan_off);
+    size_t skip_off, pre_off, plan_off, flags_off;
+    const size_t need =
+        cascade_ws_layout(S, Hkv, G, L.head_dim, P, &part_off, &skip_off, &pre_off, &plan_off, &flags_off);
     if (!workspace || ws_bytes < need || ((uintptr_t)workspace & 255u)) return KV_ERR_WORKSPACE;
     uint8_t *ws = reinterpret_cast<uint8_t *>(workspace);
     c->q = q;
@@ -547,7 +623,6 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     }
     a.ws_run = reinterpret_cast<int2 *>(ws);
     a.ws_part = reinterpret_cast<float *>(ws + part_off);
-    a.skip = c->ws_skip;
     a.chain = 2;  // beside the prefix kernel, which waits before releasing it
     a.ws_pre = c->ws_pre;
     a.KS = c->KS;
@@ -560,8 +635,31 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         if (rc) return rc;
         sync = nullptr;
     }
+    // The skips go to the skip array the previous call on this workspace did
+    // not use.  Right after that call's combine (same workspace and layout),
+    // with the pool's step overlap on, this step overlaps the combine: the
+    // plan kernel writes at once and raises its flags, the prefix kernel
+    // releases the decode kernel before its wait, and the decode kernel
+    // (chain 4) reads after the first flag and writes after the second.
+    int32_t *skip0 = reinterpret_cast<int32_t *>(ws + skip_off);
+    int32_t *skip1 = reinterpret_cast<int32_t *>(ws + skip_off + ((size_t)S * 4 + 255) / 256 * 256);
+    uint64_t *flags = reinterpret_cast<uint64_t *>(ws + flags_off);
+    KvpCascadeNote prev{};
+    const bool same_ws = kvp_stream_after_cascade(stream, &prev) && prev.ws == workspace && prev.flags == flags &&
+                         prev.plan == ws + plan_off && (prev.skip == skip0 || prev.skip == skip1);
+    c->ws_skip = same_ws && prev.skip == skip0 ? skip1 : skip0;
+    a.skip = c->ws_skip;
+    PlanOverlap ov{p->step_overlap && same_ws, flags, 0};
+    if (ov.on) {
+        p->overlapped.fetch_add(1, std::memory_order_relaxed);
+        ov.epoch = next_epoch();
+        a.chain = 4;
+        a.flags = flags;
+        a.epoch = ov.epoch;
+    }
+    c->overlap = ov.on ? 1 : 0;
     rc = cascade_plan_run(words_buf.data(), n_words, S, reinterpret_cast<int32_t *>(ws + plan_off), c->ws_skip,
-                          sync, (cudaStream_t)stream);
+                          sync, ov, (cudaStream_t)stream);
     if (rc) return rc;
     if (sync) {
         kv_seqtab *t = sync->t;
@@ -575,8 +673,11 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                   kvp::kLaunchAttention, &P);
     if (rc) return rc;
-    return dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
-                    kvp::kLaunchCombine, &P);
+    rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
+                  kvp::kLaunchCombine, &P);
+    if (rc) return rc;
+    kvp_note_cascade_combine(stream, KvpCascadeNote{workspace, a.skip, flags, ws + plan_off});
+    return KV_OK;
 }
 
 }  // namespace

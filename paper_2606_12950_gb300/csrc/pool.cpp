@@ -242,6 +242,7 @@ int kv_pool_stats(const kv_pool *p, kv_stats *out)
         out->bytes_used += (uint64_t)p->used_blocks[l] * p->block_bytes[l];
     }
     out->bytes_mapped = p->vmm.active ? p->vmm.mapped_bytes : out->bytes_total;
+    out->attn_calls_overlapped = p->overlapped.load(std::memory_order_relaxed);
     return KV_OK;
 }
 

@@ -2,6 +2,7 @@
 // (pool.cpp) and the launch wrappers (kernels.cu).  Not part of the ABI.
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <mutex>
 #include <vector>
@@ -50,6 +51,7 @@ struct kv_pool {
     int sm_count = 0;
     int attn_variant = 0;
     bool step_overlap = false;                // kv_set_attn_step_overlap
+    std::atomic<int64_t> overlapped{0};       // calls that overlapped the previous combine
     CUtensorMap tmap[KV_MAX_LAYOUTS];        // pool viewed as rows of d bf16, per layout
     bool tmap_ok[KV_MAX_LAYOUTS] = {false, false, false, false};
     kv_vmm_state vmm;

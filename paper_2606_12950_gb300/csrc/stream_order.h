@@ -15,3 +15,20 @@
 void kvp_note_stream(void *stream, bool combine);
 // true when the library's latest launch on `stream` was a split-K combine
 bool kvp_stream_after_combine(void *stream);
+
+// The workspace areas of a shared-prefix call whose combine was the latest
+// launch on a stream.  The next shared-prefix call on the same workspace
+// may then write its plan, its skips (into the other skip array) and its
+// table sync while that combine still runs: the combine reads none of them.
+struct KvpCascadeNote {
+    const void *ws;     // workspace base
+    const void *skip;   // the skip array the combine reads
+    const void *flags;  // the plan kernel's flags
+    const void *plan;   // the plan words
+};
+// mark the latest launch on `stream` (a shared-prefix call's combine) with
+// its workspace areas
+void kvp_note_cascade_combine(void *stream, const KvpCascadeNote &n);
+// true, with *n filled in, when the latest launch on `stream` was a
+// shared-prefix call's combine
+bool kvp_stream_after_cascade(void *stream, KvpCascadeNote *n);

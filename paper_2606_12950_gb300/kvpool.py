@@ -76,6 +76,7 @@ class kv_stats(ctypes.Structure):
         ("bytes_used", ctypes.c_uint64),
         ("bytes_total", ctypes.c_uint64),
         ("bytes_mapped", ctypes.c_uint64),
+        ("attn_calls_overlapped", ctypes.c_int64),
     ]
 
 
@@ -366,6 +367,7 @@ def kv_pool_stats(pool) -> dict:
         "blocks_used": list(s.blocks_used), "blocks_cached": list(s.blocks_cached),
         "blocks_capacity": list(s.blocks_capacity), "bytes_used": s.bytes_used,
         "bytes_total": s.bytes_total, "bytes_mapped": s.bytes_mapped,
+        "attn_calls_overlapped": s.attn_calls_overlapped,
     }
 
 
