@@ -15,8 +15,10 @@ stage ends, trims, releases and new chains re-sharing the prompt reach the
 plan kernel as table changes), one with the overlap on and one with it off:
 - steps back to back on one stream (the final output, lengths, table and
   pool compared: a copy between the steps would separate them);
-- an output copy and new inputs between steps (every step compared);
 - the full-size agent chains (256 chains), as the benchmark runs them;
+- 600 chains, whose plan and sync take the plan kernel's larger parameter
+  block;
+- an output copy and new inputs between steps (every step compared);
 - two batches with their own workspaces interleaved on one stream (no
   call follows a combine on its own workspace, so none overlaps).
 The pool's counter shows which calls overlapped; outputs are checked
@@ -170,6 +172,12 @@ def test_cascade_overlap_back_to_back_with_stage_turnover():
 def test_cascade_overlap_full_size_agent_chains():
     """256 chains, stage outputs lognormal(300): 12 steps back to back."""
     _back_to_back(256, steps=12, median=300.0, max_out=4096)
+
+
+def test_cascade_overlap_with_a_larger_plan():
+    """600 chains: the plan (about 1200 words) and the sync take the plan
+    kernel's 8 KB parameter block; 10 steps back to back."""
+    _back_to_back(600, steps=10, median=5.0, max_out=40, pages_per_chain=16)
 
 
 def test_cascade_overlap_with_copies_between_steps():
