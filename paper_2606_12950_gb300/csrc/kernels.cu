@@ -520,12 +520,11 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
         // right after one of this library's combines on the stream, and with
         // the pool's step overlap on, the decode grid starts while that
         // combine finishes (chain 3)
-        if (p->step_overlap && kvp_stream_after_combine(stream)) {
-            a.chain = 3;
-            p->overlapped.fetch_add(1, std::memory_order_relaxed);
-        }
+        const bool overlap = p->step_overlap && kvp_stream_after_combine(stream);
+        if (overlap) a.chain = 3;
         rc = dispatch(variant, L.head_dim, G, &p->tmap[layout], &a, num_splits, p->sm_count, (cudaStream_t)stream,
                       kvp::kLaunchBoth, &P);
+        if (rc == KV_OK && overlap) p->overlapped.fetch_add(1, std::memory_order_relaxed);
         if (rc || !sync) return rc;
         kv_seqtab *t = sync->t;
         t->counters.entries_uploaded += (int64_t)t->changed.size();
@@ -651,7 +650,6 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
     a.skip = c->ws_skip;
     PlanOverlap ov{p->step_overlap && same_ws, flags, 0};
     if (ov.on) {
-        p->overlapped.fetch_add(1, std::memory_order_relaxed);
         ov.epoch = next_epoch();
         a.chain = 4;
         a.flags = flags;
@@ -677,6 +675,7 @@ int attn_call(kv_pool *p, int layout, const uint16_t *q, const uint16_t *k_new, 
                   kvp::kLaunchCombine, &P);
     if (rc) return rc;
     kvp_note_cascade_combine(stream, KvpCascadeNote{workspace, a.skip, flags, ws + plan_off});
+    if (ov.on) p->overlapped.fetch_add(1, std::memory_order_relaxed);
     return KV_OK;
 }
 
