@@ -19,6 +19,8 @@ plan kernel as table changes), one with the overlap on and one with it off:
 - 600 chains, whose plan and sync take the plan kernel's larger parameter
   block;
 - an output copy and new inputs between steps (every step compared);
+- the pool's error word read between some steps (a library copy: the next
+  call does not overlap);
 - two batches with their own workspaces interleaved on one stream (no
   call follows a combine on its own workspace, so none overlaps).
 The pool's counter shows which calls overlapped; outputs are checked
@@ -201,6 +203,34 @@ def test_cascade_overlap_with_copies_between_steps():
     for i, (x, y) in enumerate(zip(res["on"], res["off"])):
         _equal(x, y, f"step {i}")
     assert on.overlapped() - on.overlapped0 == on.expected_overlaps() >= steps // 2
+    on.mirror()
+    assert np.array_equal(on.pool.download(), on.host_pool)
+    on.close()
+    off.close()
+
+
+def test_cascade_overlap_off_after_a_library_copy():
+    """The pool's error word read (a copy and a clear by the library) after
+    every third step: the call after it waits for the combine instead of
+    overlapping it; the bits still match the overlap off, and the final
+    output matches the oracle."""
+    steps = 15
+    on = Side(48, 5.0, 40, True)
+    off = Side(48, 5.0, 40, False)
+    for side in (on, off):
+        after_copy = []
+        for i in range(steps):
+            after_copy.append(i > 0 and (i - 1) % 3 == 2)
+            table, lens = side.step()
+            if i % 3 == 2:
+                assert side.pool.error() == 0
+        torch.cuda.synchronize()
+        side.final = (table, lens)
+    _equal(on.bits(), off.bits(), "final output, lengths and table")
+    expected = sum(1 for i in range(1, steps) if not on.separate[i] and not after_copy[i])
+    assert expected >= steps // 2
+    assert on.overlapped() - on.overlapped0 == expected
+    on.check(*on.final, "final step, overlap on")
     on.mirror()
     assert np.array_equal(on.pool.download(), on.host_pool)
     on.close()
