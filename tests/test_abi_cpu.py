@@ -118,6 +118,20 @@ def test_free_and_ref_validation_changes_nothing():
     K.kv_pool_destroy(h)
 
 
+def test_stats_of_a_fresh_pool():
+    """kv_stats as the binding reads it: a fresh pool's pages, bytes and its
+    count of overlapped attention calls (the last field: a layout mismatch
+    between the header and the binding shows here)."""
+    h, _ = make_pool(n_pages=16)
+    st = K.kv_pool_stats(h)
+    assert st["pages_total"] == 16
+    assert st["bytes_used"] == 0 and st["bytes_mapped"] == st["bytes_total"] > 0
+    assert st["attn_calls_overlapped"] == 0
+    K.kv_set_attn_step_overlap(h, 1)
+    assert K.kv_pool_stats(h)["attn_calls_overlapped"] == 0
+    K.kv_pool_destroy(h)
+
+
 def test_shuffled_free_order_is_a_seeded_permutation():
     h1, _ = make_pool(n_pages=256, seed=42)
     h2, _ = make_pool(n_pages=256, seed=42)
